@@ -1,0 +1,466 @@
+#!/usr/bin/env python3
+"""Benchmark of the restoration sweep (fingerprint, pack, unpack+verify, diff).
+
+One step is one restoration of a rank's state from a data-parallel replica
+(FlashRecovery, arXiv 2509.03047, Sec. III-E), with every sweep call once:
+  fingerprint(replica) -> pack(replica -> transfer buffer) -> inject the
+  workload's bit flips -> unpack_verify(buffer -> restored rank)
+  -> fingerprint(restored) -> diff(tables).
+The default workload is the largest one that fits one GPU: a Llama-3-70B
+rank at TP=8/PP=4 (20 layers + embedding, bf16 weight + fp32 master/m/v,
+31.8 GB), 16 MiB chunks, 50 NaNs in the state and 1,000 bit flips in the
+buffer.  Inputs are synthetic and seeded, and far larger than L2.
+
+value = state bytes swept per step (4 sweeps of S) / step time, in GB/s,
+summed over ranks (replicas only: every rank restores its own state; no
+collective is on the data path).
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl flashrec|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "state GB/s per call (fingerprint, pack, unpack+verify) and fraction of HBM peak"
+SWEEPS_PER_STEP = 4  # fingerprint x2, pack, unpack_verify each touch every state byte
+DEFAULT_CONFIG = "l70b_tp8pp4"
+
+
+# ---------------------------------------------------------------- distributed plumbing
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def dist_setup(backend: str):
+    import torch.distributed as dist
+
+    ws, rank, _ = dist_env()
+    if ws > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        os.environ.setdefault("MASTER_PORT", "29511")
+        dist.init_process_group(backend=backend, rank=rank, world_size=ws)
+    return ws, rank
+
+
+def barrier():
+    import torch.distributed as dist
+
+    if dist.is_initialized():
+        dist.barrier()
+
+
+def max_over_ranks(x: float, device=None) -> float:
+    import torch
+    import torch.distributed as dist
+
+    if not dist.is_initialized():
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x: float, device=None) -> float:
+    import torch
+    import torch.distributed as dist
+
+    if not dist.is_initialized():
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        return self.summary()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- helpers
+
+def measured_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def profiled_traffic(kernel_key: str, workload: str):
+    """DRAM bytes per launch of `kernel_key` from a committed ncu summary, if
+    it was taken on the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    from paper_2509_03047_gb300 import build as _b
+
+    ent = rec.get(kernel_key)
+    if not ent or ent.get("workload") != workload or ent.get("sources") != _b.source_digest():
+        return None
+    return ent.get("bytes_per_launch")
+
+
+def sweep_classes(tensors):
+    """Sweep kernels a call launches: one per (element type, 16-byte aligned)
+    class that has a chunk body (the library's own planning rule)."""
+    from paper_2509_03047_gb300 import flashrec as fr
+
+    cls = set()
+    for t in tensors:
+        if t.numel() * t.element_size() >= 512:
+            cls.add((fr.fr_dtype_of(t), t.data_ptr() % 16 == 0))
+    return len(cls)
+
+
+# ---------------------------------------------------------------- the flashrec arm
+
+def run_flashrec(args):
+    import numpy as np
+    import torch
+
+    from paper_2509_03047_gb300 import flashrec as fr
+    from paper_2509_03047_gb300 import synth
+
+    ws, rank = dist_setup("nccl")
+    _, _, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    cfg = synth.get_config(args.config)
+    src = synth.make_state(cfg, dev)
+    nan_pos = synth.inject_nonfinite(cfg, src)
+    dst = [torch.empty_like(t) for t in src]
+    plan_s = fr.Plan(src, cfg.chunk_bytes)
+    plan_d = fr.Plan(dst, cfg.chunk_bytes)
+    S, C, P = plan_s.state_bytes, plan_s.n_chunks, plan_s.packed_bytes
+    packed = plan_s.new_packed()
+    tab_s, tab_d = plan_s.new_table(), plan_d.new_table()
+    mism = torch.empty(C, dtype=torch.int32, device=dev)
+    nmis = torch.empty(1, dtype=torch.int64, device=dev)
+    div = torch.empty(C, dtype=torch.int32, device=dev)
+    ndiv = torch.empty(1, dtype=torch.int64, device=dev)
+    flips = synth.flip_positions(P, cfg.flips, cfg.seed)
+    fb = np.unique(flips // 8)
+    fmask = np.zeros(fb.size, dtype=np.uint8)
+    for p in flips:
+        fmask[np.searchsorted(fb, p // 8)] ^= np.uint8(1 << (p % 8))
+    flip_idx = torch.as_tensor(fb, dtype=torch.int64, device=dev)
+    flip_mask = torch.as_tensor(fmask, device=dev)
+    flip_idx_h = torch.as_tensor(fb, dtype=torch.int64)
+    flip_mask_h = torch.as_tensor(fmask)
+    stream = torch.cuda.current_stream()
+    n_cls = sweep_classes(src)
+
+    def step(ev=None, buf=packed, sync_counts=False):
+        if ev:
+            ev[0].record(stream)
+        fr.fr_fingerprint(plan_s.handle, tab_s, stream)
+        if ev:
+            ev[1].record(stream)
+        fr.fr_pack(plan_s.handle, buf, stream)
+        if ev:
+            ev[2].record(stream)
+        if flip_idx.numel():  # the workload's faults in the transfer buffer
+            if buf.is_cuda:
+                buf[flip_idx] ^= flip_mask
+            else:
+                stream.synchronize()
+                buf[flip_idx_h] ^= flip_mask_h
+        if ev:
+            ev[3].record(stream)
+        fr.fr_unpack_verify(plan_d.handle, buf, mism, nmis, stream)
+        if ev:
+            ev[4].record(stream)
+        fr.fr_fingerprint(plan_d.handle, tab_d, stream)
+        if ev:
+            ev[5].record(stream)
+        fr.fr_diff(tab_s, tab_d, C, div, ndiv, stream)
+        if ev:
+            ev[6].record(stream)
+        if sync_counts:
+            return int(nmis.item()), int(ndiv.item())
+        return None
+
+    launches_per_step = (n_cls + 1) * 2 + (n_cls + 1) + (n_cls + 2) + 1
+
+    # correctness of the timed configuration: the injected flips are found
+    for _ in range(args.warmup):
+        step()
+    n_mis, n_div = step(sync_counts=True)
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(args.steps)]
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for k in range(args.steps):
+        step(evs[k])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    names = ["fingerprint_replica", "pack", "inject_flips", "unpack_verify", "fingerprint_restored", "diff"]
+    per = {n: sum(e[i].elapsed_time(e[i + 1]) for e in evs) / args.steps for i, n in enumerate(names)}
+    ms_step = max_over_ranks(total_ms / args.steps, dev)
+    value = sum_over_ranks(SWEEPS_PER_STEP * S / (ms_step * 1e-3) / 1e9, dev)
+
+    # ---- roofline of the dominant kernel pair (sweep + finalize of one call)
+    peak, peak_kind = measured_peak()
+    H = P - S  # header table, gap and padding bytes
+    alg = {"fingerprint": S + 16 * C, "pack": S + P, "unpack_verify": P + S + 4 * C}
+    t_call = {"fingerprint": (per["fingerprint_replica"] + per["fingerprint_restored"]) / 2,
+              "pack": per["pack"], "unpack_verify": per["unpack_verify"]}
+    share = {"fingerprint": 2 * t_call["fingerprint"], "pack": t_call["pack"],
+             "unpack_verify": t_call["unpack_verify"]}
+    dom = max(share, key=share.get)
+    calls = {}
+    for k in alg:
+        gbs = alg[k] / (t_call[k] * 1e-3) / 1e9
+        calls[k] = {"ms": round(t_call[k], 4), "state_gbs": round(S / (t_call[k] * 1e-3) / 1e9, 1),
+                    "alg_bytes": alg[k], "achieved_gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
+                    "frac_of_8tbs": round(gbs / 8000.0, 4)}
+    calls["diff"] = {"us": round(per["diff"] * 1e3, 2), "alg_bytes": 32 * C}
+    calls["inject_flips_us"] = round(per["inject_flips"] * 1e3, 2)
+    ach = alg[dom] / (t_call[dom] * 1e-3) / 1e9
+    roofline = {"kernel": "fr_%s (sweep + finalize kernels)" % dom, "bound": "hbm", "achieved": round(ach, 1),
+                "peak": peak, "unit": "GB/s", "frac": round(ach / peak, 4),
+                "peak_source": "%s HBM copy bandwidth (MEASURED_PEAKS.json hbm_gbs)" % peak_kind
+                if peak_kind == "measured" else "fallback 6.8 TB/s",
+                "traffic": profiled_traffic("fr_" + dom, args.config),
+                "alg_bytes_per_launch": alg[dom]}
+
+    # ---- end to end through the C ABI with the transfer buffer in pinned host memory
+    e2e = None
+    if not args.no_e2e:
+        host_buf = plan_s.new_packed(pinned=True)
+        step(buf=host_buf, sync_counts=True)
+        barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            step(buf=host_buf, sync_counts=True)  # D2H pack, H2D unpack, D2H counts
+        torch.cuda.synchronize()
+        t_e2e = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
+        e2e = {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_e2e / 1e9, dev), 2), "unit": "GB/s",
+               "h2d_bytes_per_step": P, "d2h_bytes_per_step": P + 16, "ms_per_step": round(t_e2e * 1e3, 2),
+               "transfer": "pinned host buffer over NVLink-C2C, written and read by the kernels"}
+        del host_buf
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(cfg, src, args.cpu_sample_gb)
+
+    if rank == 0:
+        out = {"metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
+               "warmup": args.warmup, "ms_per_step": round(ms_step, 3), "higher_is_better": True,
+               "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+               "data": "synthetic (seeded; shapes of the named model shard)",
+               "config": {"workload": args.config, "state_bytes": S, "chunk_bytes": cfg.chunk_bytes,
+                          "n_chunks": C, "packed_bytes": P, "header_pad_bytes": H,
+                          "faults": {"nan": int(nan_pos.size), "bit_flips": int(flips.size)},
+                          "found": {"mismatching_chunks": n_mis, "diverged_chunks": n_div},
+                          "l2": "inputs larger than L2 (state %.1f GB vs 129 MB L2); no flush" % (S / 1e9),
+                          "parallelism": "replicas only (%d independent rank%s)" % (ws, "s" if ws > 1 else ""),
+                          "value_def": "4 sweeps x state bytes / step time"},
+               "calls": calls, "roofline": roofline, "e2e": e2e, "cpu_baseline": cpu,
+               "gpu_launches": launches_per_step * args.steps, "clocks": clk}
+        print(json.dumps(out))
+    plan_s.close()
+    plan_d.close()
+
+
+# ---------------------------------------------------------------- the oracle
+
+def oracle_sample(cfg, tensors_host, dtypes, steps=1):
+    """Time the CPU oracle doing one restoration step on a host sample."""
+    import oracle
+
+    oracle.build()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        fa = oracle.fingerprint(tensors_host, dtypes, cfg.chunk_bytes)
+        pk = oracle.pack(tensors_host, dtypes, cfg.chunk_bytes)
+        dst = [h.copy() for h in tensors_host]
+        oracle.unpack_verify(dst, dtypes, cfg.chunk_bytes, pk)
+        fb = oracle.fingerprint(dst, dtypes, cfg.chunk_bytes)
+        oracle.diff(fa, fb)
+    return (time.perf_counter() - t0) / steps
+
+
+def sample_buffers(cfg, sample_gb):
+    """Indices of a bounded, representative slice of the state's buffers:
+    whole parameter groups (weight, master, m, v) in order, skipping any single
+    parameter larger than the budget (the embedding), so the bf16/fp32 mix is
+    the workload's; for the fragmented state, its first buffers."""
+    limit = int(sample_gb * 1e9)
+    specs = cfg.buffer_specs()
+    idx, tot = [], 0
+    group = 4 if cfg.kind == "adam" else 1
+    for g in range(0, len(specs), group):
+        nb = sum(b for _, _, b in specs[g:g + group])
+        if nb > limit and not idx:
+            continue
+        if idx and tot + nb > limit:
+            break
+        idx += list(range(g, g + group))
+        tot += nb
+    return idx, tot
+
+
+def cpu_baseline(cfg, tensors, sample_gb):
+    import torch
+
+    from paper_2509_03047_gb300 import flashrec as fr
+
+    idx, tot = sample_buffers(cfg, sample_gb)
+    host = [tensors[i].view(torch.uint8).reshape(-1).cpu().numpy() for i in idx]
+    dts = [fr.fr_dtype_of(tensors[i]) for i in idx]
+    dt = oracle_sample(cfg, host, dts)
+    return {"value": round(SWEEPS_PER_STEP * tot / dt / 1e9, 4), "unit": "GB/s", "cores": 1,
+            "host_cores": os.cpu_count(), "kind": "oracle",
+            "sample": "%d buffers (%.2f GB) of the %s state, one restoration step (fingerprint, pack, "
+                      "unpack_verify, fingerprint, diff), single thread, %.1f s" % (len(host), tot / 1e9,
+                                                                                    cfg.name, dt)}
+
+
+def run_reference(args):
+    """The reference arm: the CPU oracle as it stands, on the host cores, on a
+    bounded slice of the same workload generated on the host."""
+    import torch
+
+    from paper_2509_03047_gb300 import synth
+    from paper_2509_03047_gb300.flashrec import FR_DT_BF16, FR_DT_F32
+
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return
+    cfg = synth.get_config(args.config)
+    idx, tot = sample_buffers(cfg, args.cpu_sample_gb)
+    if cfg.kind == "adam":
+        sub = synth.Config(cfg.name, cfg.chunk_bytes, "adam", [cfg.shapes[i // 4] for i in idx[::4]],
+                           seed=cfg.seed)
+        state = synth.make_state(sub, "cpu")
+    else:
+        specs = cfg.buffer_specs()
+        state = [torch.randn(specs[i][2] // 4, generator=synth._gen("cpu", cfg.seed, i, 9)) for i in idx]
+    host = [t.view(torch.uint8).reshape(-1).numpy() for t in state]
+    dts = [FR_DT_BF16 if t.dtype == torch.bfloat16 else FR_DT_F32 for t in state]
+    times = [oracle_sample(cfg, host, dts) for _ in range(args.steps)]
+    dt = sum(times) / len(times)
+    value = SWEEPS_PER_STEP * tot / dt / 1e9
+    cpu = {"value": round(value, 4), "unit": "GB/s", "cores": 1, "host_cores": os.cpu_count(), "kind": "oracle",
+           "sample": "%d buffers (%.2f GB) of the %s state per step, single thread" % (len(host), tot / 1e9,
+                                                                                     cfg.name)}
+    out = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": ws,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 1),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+           "data": "synthetic (seeded; shapes of the named model shard)",
+           "config": {"workload": args.config, "sample_bytes": tot, "chunk_bytes": cfg.chunk_bytes,
+                      "value_def": "4 sweeps x state bytes / step time"},
+           "cpu_baseline": cpu,
+           "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["flashrec", "reference"], default="flashrec")
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-gb", type=float, default=1.0)
+    args = ap.parse_args(argv)
+    if args.warmup < 3 and args.impl == "flashrec":
+        ap.error("at least 3 warm-up steps")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_flashrec(args)
+
+
+if __name__ == "__main__":
+    main()

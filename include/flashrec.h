@@ -1,0 +1,174 @@
+/*
+ * flashrec.h -- C ABI of libflashrec, the GB300 (sm_103a) restoration sweep.
+ *
+ * FlashRecovery (arXiv 2509.03047) restores a restarted rank's model and
+ * optimizer state from a healthy data-parallel replica's memory instead of
+ * from a checkpoint (Sec. III-E, "Model states Restoration"; vanilla-DP panel
+ * of the restoration figure).  The paper moves the state "with collective
+ * communication" and defines no checksum or transfer format.  This library is
+ * the device-side sweep over one rank's state that such a restoration needs:
+ *
+ *   fr_fingerprint    per-chunk CRC-32C, non-finite count, fp64 sum of squares
+ *   fr_pack           tensors -> one flat transfer buffer with chunk headers
+ *   fr_unpack_verify  transfer buffer -> tensors, list of failing chunks
+ *   fr_diff           chunks whose fingerprints differ
+ *
+ * All device work runs in hand-written CUDA kernels for sm_103a.  There is no
+ * CPU fallback: without a usable GPU every call returns FR_ERR_CUDA.
+ *
+ * Conventions
+ *   - Chunks are per tensor: chunk k of tensor t covers bytes
+ *     [k*chunk_bytes, min((k+1)*chunk_bytes, nbytes_t)).  Chunk ids are global
+ *     and ascending in tensor order, then offset.  A 0-byte tensor has no chunk.
+ *   - CRC-32C: polynomial 0x1EDC6F41 (reflected 0x82F63B78), reflected in and
+ *     out, preset 0xFFFFFFFF, final XOR 0xFFFFFFFF (CRC-32/ISCSI).
+ *   - An element is non-finite when its exponent field is all ones.  sumsq is
+ *     the sum of x*x over the finite elements, accumulated in fp64; it agrees
+ *     with a sequential fp64 sum to within 1e-9 relative and is bit-for-bit
+ *     reproducible from run to run on the same GPU.
+ *   - Every device call is asynchronous and ordered on `stream` (a
+ *     cudaStream_t passed as void*; NULL is the legacy default stream).
+ *     Argument errors are returned synchronously and enqueue nothing.
+ *     Conditions found on the device (list overflow) are recorded in the plan
+ *     and returned by fr_sync_status().
+ *   - Pointers named *_dev are device memory (or any memory the GPU can
+ *     address through unified virtual addressing, such as pinned host memory).
+ *     The caller owns every tensor, buffer and output; the library owns only
+ *     the plan and what the plan allocates when it is created.  No call after
+ *     fr_plan_create allocates memory.
+ *   - Thread safety: a plan may be used by one stream at a time.
+ */
+#ifndef FLASHREC_H
+#define FLASHREC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  FR_OK = 0,
+  FR_ERR_INVALID_ARG = 1,      /* a null pointer, bad dtype, size or chunk size  */
+  FR_ERR_ALIGNMENT = 2,        /* the packed buffer is not 16-byte aligned       */
+  FR_ERR_BUFFER_TOO_SMALL = 3, /* the packed buffer is shorter than the plan's   */
+  FR_ERR_CAPACITY = 4,         /* more ids than the list holds (true count kept) */
+  FR_ERR_PLAN_MISMATCH = 5,    /* a table length that differs from the plan's    */
+  FR_ERR_DEVICE_TIMEOUT = 6,   /* a bounded device-side wait gave up             */
+  FR_ERR_CUDA = 7              /* a CUDA runtime error; see fr_last_error()      */
+} fr_status;
+
+typedef enum {
+  FR_DT_BYTES = 0, /* opaque bytes: CRC only, nonfinite = 0, sumsq = 0 */
+  FR_DT_BF16 = 1,
+  FR_DT_F32 = 2
+} fr_dtype;
+
+/* One tensor of the state: `nbytes` bytes of device memory at `ptr`
+ * (any alignment; 16-byte-aligned tensors take the fast path).  nbytes must
+ * be a multiple of the element size.  `flags` must be 0. */
+typedef struct {
+  void* ptr;
+  uint64_t nbytes;
+  uint32_t dtype;
+  uint32_t flags;
+} fr_tensor;
+
+/* One fingerprint table entry: 16 bytes, no padding. */
+typedef struct {
+  uint32_t crc32c;    /* CRC-32C of the chunk's bytes                 */
+  uint32_t nonfinite; /* elements whose exponent field is all ones     */
+  double sumsq;       /* sum of squares of the finite elements (fp64)  */
+} fr_fp;
+
+typedef struct fr_plan_s* fr_plan;
+
+/* ---------------------------------------------------------------- plans */
+
+/* Build a plan over `n_tensors` tensors (host array, copied) with chunks of
+ * `chunk_bytes` (a positive multiple of 4).  The plan is bound to the current
+ * CUDA device and to the tensors' addresses; it allocates its device tables
+ * and scratch here and nowhere else.  Host-side planning is O(tensors +
+ * chunks).  Errors: FR_ERR_INVALID_ARG, FR_ERR_CUDA. */
+fr_status fr_plan_create(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes,
+                         fr_plan* out);
+
+/* Chunk count, packed buffer size and total state bytes of a plan (host). */
+fr_status fr_plan_info(fr_plan plan, uint64_t* n_chunks, uint64_t* packed_bytes,
+                       uint64_t* state_bytes);
+
+/* Where chunk `chunk_id` lives (host query): its tensor, byte offset in the
+ * tensor, length, and payload offset in the packed buffer. */
+fr_status fr_plan_chunk(fr_plan plan, uint64_t chunk_id, uint32_t* tensor_idx,
+                        uint64_t* tensor_off, uint64_t* len, uint64_t* payload_off);
+
+/* Free the plan and its device memory (synchronizes the device first). */
+void fr_plan_destroy(fr_plan plan);
+
+/* ---------------------------------------------------------------- sweep */
+
+/* Fingerprint every chunk of the plan's tensors into `out_dev`, an array of
+ * n_chunks fr_fp entries.  Restoration step of Sec. III-E: the table a healthy
+ * replica and a restored rank compare.  Reads the state once. */
+fr_status fr_fingerprint(fr_plan plan, fr_fp* out_dev, void* stream);
+
+/* Gather the plan's tensors into the transfer buffer `dst` (device memory or
+ * pinned host memory; 16-byte aligned; at least packed_bytes long), the
+ * replica side of the Sec. III-E restoration.  Layout (little-endian):
+ *   [n_chunks x 64-byte headers][zero bytes to a 256-byte boundary]
+ *   then each chunk's payload at a 256-byte-aligned offset, zero-padded to
+ *   the next 256-byte boundary.
+ * Header: 0 u32 magic 'FRC1' | 4 u16 version 1 | 6 u16 dtype | 8 u64 chunk_id
+ *   | 16 u32 tensor_idx | 20 u32 payload_crc | 24 u64 tensor_off | 32 u64 len
+ *   | 40 u64 payload_off | 48 f64 sumsq | 56 u32 nonfinite
+ *   | 60 u32 header_crc = CRC-32C of bytes [0,60).
+ * Every byte of [0, packed_bytes) is written.
+ * Errors: FR_ERR_INVALID_ARG, FR_ERR_ALIGNMENT, FR_ERR_BUFFER_TOO_SMALL, FR_ERR_CUDA. */
+fr_status fr_pack(fr_plan plan, void* dst, uint64_t dst_bytes, void* stream);
+
+/* Scatter the transfer buffer `src` (device or pinned host; 16-byte aligned)
+ * into the plan's tensors, the restarted-rank side of Sec. III-E.  Every
+ * payload is copied to the address the receiver's own plan gives (a header is
+ * never trusted for addressing).  A chunk is listed when its header CRC is
+ * wrong, any header field differs from the plan (magic, version, dtype,
+ * chunk_id, tensor_idx, tensor_off, len, payload_off), its payload CRC-32C
+ * differs from the header's payload_crc, or a padding byte after its payload
+ * is non-zero (the zero bytes after the header table belong to the last
+ * chunk).  The ids go to `mismatch_dev` in ascending order, at most `cap` of
+ * them; the true count goes to *n_mismatch_dev (device u64).  When the count
+ * exceeds `cap` the plan records FR_ERR_CAPACITY for fr_sync_status().
+ * Errors: FR_ERR_INVALID_ARG, FR_ERR_ALIGNMENT, FR_ERR_BUFFER_TOO_SMALL, FR_ERR_CUDA. */
+fr_status fr_unpack_verify(fr_plan plan, const void* src, uint64_t src_bytes,
+                           uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev,
+                           void* stream);
+
+/* Chunks whose 16-byte table entries differ in any bit (crc32c, nonfinite, or
+ * the bit pattern of sumsq) between `a_dev` and `b_dev`, both n_chunks long.
+ * Ascending ids, at most `cap`, to `diverged_dev`; the true count to
+ * *n_out_dev (device u64).  Overflow is visible as count > cap.
+ * Errors: FR_ERR_INVALID_ARG, FR_ERR_CUDA. */
+fr_status fr_diff(const fr_fp* a_dev, const fr_fp* b_dev, uint64_t n_chunks,
+                  uint32_t* diverged_dev, uint64_t cap, uint64_t* n_out_dev, void* stream);
+
+/* ---------------------------------------------------------------- status */
+
+/* Synchronize `stream`, then return and clear the first condition the plan's
+ * kernels recorded (FR_ERR_CAPACITY or FR_ERR_DEVICE_TIMEOUT), else FR_OK. */
+fr_status fr_sync_status(fr_plan plan, void* stream);
+
+/* A static string naming a status code. */
+const char* fr_status_str(fr_status status);
+
+/* The message of the last FR_ERR_CUDA / FR_ERR_INVALID_ARG seen by the
+ * calling thread ("" if none). */
+const char* fr_last_error(void);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int fr_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FLASHREC_H */

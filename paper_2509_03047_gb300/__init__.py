@@ -1,0 +1,8 @@
+"""libflashrec for GB300 (sm_103a): the restoration sweep of FlashRecovery
+(arXiv 2509.03047, Sec. III-E) -- per-chunk fingerprint, pack, unpack+verify
+and diff over a rank's model and optimizer state, in hand-written CUDA.
+
+``paper_2509_03047_gb300.flashrec`` is the ctypes binding of the C ABI in
+``include/flashrec.h``; importing it fails loudly if the library is not built.
+``paper_2509_03047_gb300.synth`` generates the seeded synthetic workloads.
+"""

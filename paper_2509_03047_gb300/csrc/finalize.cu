@@ -1,0 +1,362 @@
+// finalize.cu -- per-chunk fold, tails, headers and verification; ordered
+// compaction of chunk ids; fingerprint diff.
+//
+// The sweep kernel leaves one record per piece (the part of a chunk body one
+// warp covered).  Here one warp per chunk:
+//   1. shifts each record's raw CRC to its position in the chunk and XORs them
+//      (raw(A||B) = raw(A) * x^(8|B|) ^ raw(B)), and sums the records' sums of
+//      squares and non-finite counts in record order;
+//   2. handles the chunk's tail (len % 512 bytes): lane l takes bytes
+//      [16l, 16l+16) of it, CRCs them a byte at a time, sums their squares in
+//      fp64, and copies them for pack/unpack;
+//   3. applies CRC-32C's preset and final XOR:
+//      crc = raw ^ 0xFFFFFFFF * x^(8 len) ^ 0xFFFFFFFF;
+//   4. fingerprint: writes the table entry; pack: writes the 64-byte header,
+//      the zero padding after the payload and, for the last chunk, the zero gap
+//      after the header table; unpack: checks the header against the plan, the
+//      header CRC, the payload CRC and the padding, and writes a verdict.
+// The verdicts become an ascending id list through a single-CTA ordered
+// compaction, which fr_diff shares with a different predicate.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "gf2.cuh"
+#include "kernels.h"
+#include "layout.h"
+
+namespace frk {
+
+namespace {
+
+constexpr int kFinWarps = 8;
+constexpr int kFinThreads = kFinWarps * 32;
+constexpr unsigned kFull = 0xFFFFFFFFu;
+
+__device__ const ByteTable g_byte = make_byte_table();
+__device__ const PowTables g_pow = make_pow_tables();
+
+// a * b mod P, both variable.
+__device__ __forceinline__ uint32_t gmul(uint32_t a, uint32_t b) {
+  uint32_t r = 0;
+#pragma unroll 8
+  for (int k = 0; k < 32; ++k) {
+    r ^= b & static_cast<uint32_t>(static_cast<int32_t>(a << k) >> 31);
+    b = (b >> 1) ^ (kPoly & (0u - (b & 1u)));
+  }
+  return r;
+}
+
+// x^(8n) mod P for n < 2^48, from per-byte power tables.
+__device__ uint32_t xpow8(uint64_t n) {
+  uint32_t r = kOne;
+  for (int k = 0; k < kPowBytes; ++k) {
+    const uint32_t byte = static_cast<uint32_t>(n >> (8 * k)) & 255u;
+    if (byte) r = gmul(r, __ldg(&g_pow.p[k][byte]));
+  }
+  return r;
+}
+
+__device__ __forceinline__ uint32_t shift_bytes(uint32_t raw, uint64_t n) {
+  return n ? gmul(raw, xpow8(n)) : raw;
+}
+
+__device__ __forceinline__ uint32_t crc_byte(const uint32_t* T, uint32_t r, uint32_t b) {
+  return T[(r ^ b) & 0xFFu] ^ (r >> 8);
+}
+
+__device__ __forceinline__ void exact_elem(uint32_t dtype, uint32_t bits, uint32_t& nf, double& s) {
+  if (dtype == kDtF32) {
+    if ((bits & 0x7F800000u) == 0x7F800000u) {
+      ++nf;
+    } else {
+      const double x = static_cast<double>(__uint_as_float(bits));
+      s = __dadd_rn(s, __dmul_rn(x, x));
+    }
+  } else {
+    if ((bits & 0x7F80u) == 0x7F80u) {
+      ++nf;
+    } else {
+      const double x = static_cast<double>(__uint_as_float(bits << 16));
+      s = __dadd_rn(s, __dmul_rn(x, x));
+    }
+  }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p) {
+  __shared__ uint32_t T[256];
+  for (int i = threadIdx.x; i < 256; i += kFinThreads) T[i] = g_byte.t[i];
+  __syncthreads();
+  const uint32_t lane = threadIdx.x & 31u;
+  const uint64_t stride = static_cast<uint64_t>(gridDim.x) * kFinWarps;
+  for (uint64_t c = static_cast<uint64_t>(blockIdx.x) * kFinWarps + (threadIdx.x >> 5); c < p.n_chunks;
+       c += stride) {
+    const ChunkDesc cd = p.chunks[c];
+    const uint64_t body = cd.len & ~static_cast<uint64_t>(kBlockBytes - 1);
+    const uint32_t tail = static_cast<uint32_t>(cd.len - body);
+    const bool values = (MODE != kModeUnpack) && (cd.dtype != kDtBytes);
+
+    // ---- 1. records, last batch first so the byte count after each is known
+    uint32_t raw = 0;
+    double sq_rec = 0.0;
+    uint32_t nf_rec = 0;
+    uint64_t carry = tail;
+    for (int64_t hi = cd.n_recs; hi > 0;) {
+      const int64_t lo = hi > 32 ? hi - 32 : 0;
+      const int64_t i = lo + lane;
+      const bool have = i < hi;
+      Record rec{0u, 0u, 0.0};
+      uint64_t len = 0;
+      if (have) {
+        rec = p.recs[cd.first_rec + i];
+        len = p.rec_nblk[cd.first_rec + i] * kBlockBytes;
+      }
+      uint64_t suf = len;  // bytes of this record and the later ones in the batch
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const uint64_t t = __shfl_down_sync(kFull, suf, d);
+        if (lane + d < 32) suf += t;
+      }
+      if (have) raw ^= shift_bytes(rec.crc, carry + suf - len);
+      carry += __shfl_sync(kFull, suf, 0);
+      double s = rec.sumsq;
+      uint32_t n = rec.nonfinite;
+#pragma unroll
+      for (int m = 16; m >= 1; m >>= 1) {
+        s += __shfl_down_sync(kFull, s, m);
+        n += __shfl_down_sync(kFull, n, m);
+      }
+      sq_rec += __shfl_sync(kFull, s, 0);
+      nf_rec += __shfl_sync(kFull, n, 0);
+      hi = lo;
+    }
+
+    // ---- 2. tail
+    const uint8_t* tsrc;
+    uint8_t* tdst = nullptr;
+    if (MODE == kModeUnpack) {
+      tsrc = p.packed + cd.payload_off + body;
+      tdst = reinterpret_cast<uint8_t*>(cd.addr) + body;
+    } else {
+      tsrc = reinterpret_cast<const uint8_t*>(cd.addr) + body;
+      if (MODE == kModePack) tdst = p.packed + cd.payload_off + body;
+    }
+    double sq_tail = 0.0;
+    uint32_t nf_tail = 0;
+    const uint32_t b0 = lane * 16u;
+    if (b0 < tail) {
+      const uint32_t b1 = (b0 + 16u < tail) ? b0 + 16u : tail;
+      uint32_t r = 0, word = 0;
+      for (uint32_t j = b0; j < b1; ++j) {
+        const uint32_t v = __ldg(tsrc + j);
+        r = crc_byte(T, r, v);
+        if (tdst) tdst[j] = static_cast<uint8_t>(v);
+        word |= v << (8 * (j & 3u));
+        if (values) {
+          if (cd.dtype == kDtF32 && (j & 3u) == 3u) {
+            exact_elem(kDtF32, word, nf_tail, sq_tail);
+            word = 0;
+          } else if (cd.dtype == kDtBf16 && (j & 1u) == 1u) {
+            exact_elem(kDtBf16, word >> (8 * ((j - 1) & 3u)), nf_tail, sq_tail);
+            if ((j & 3u) == 3u) word = 0;
+          }
+        }
+      }
+      raw ^= shift_bytes(r, tail - b1);
+    }
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) {
+      raw ^= __shfl_xor_sync(kFull, raw, m);
+      sq_tail += __shfl_down_sync(kFull, sq_tail, m);
+      nf_tail += __shfl_down_sync(kFull, nf_tail, m);
+    }
+
+    // ---- 3. preset and final XOR
+    const uint32_t crc = raw ^ shift_bytes(0xFFFFFFFFu, cd.len) ^ 0xFFFFFFFFu;
+    const double sumsq = sq_rec + sq_tail;  // lane 0 holds the fixed-order sums
+    const uint32_t nonfinite = nf_rec + nf_tail;
+
+    const uint64_t pad_begin = cd.payload_off + cd.len;
+    const uint64_t pad_end = cd.payload_off + align_up(cd.len, kPayloadAlign);
+    const uint64_t table_end = p.n_chunks * kHeaderBytes;
+    const uint64_t gap_end = align_up(table_end, kPayloadAlign);
+    const bool last = (c + 1 == p.n_chunks);
+
+    // ---- 4. outputs
+    if (MODE == kModeFingerprint) {
+      if (lane == 0) {
+        FpEntry e;
+        e.crc32c = crc;
+        e.nonfinite = nonfinite;
+        e.sumsq = sumsq;
+        p.out_fp[c] = e;
+      }
+    } else if (MODE == kModePack) {
+      if (lane == 0) {
+        uint32_t h[16];
+        const uint64_t sbits = static_cast<uint64_t>(__double_as_longlong(sumsq));
+        h[0] = kMagic;
+        h[1] = kVersion | (cd.dtype << 16);
+        h[2] = static_cast<uint32_t>(c);
+        h[3] = static_cast<uint32_t>(c >> 32);
+        h[4] = cd.tensor_idx;
+        h[5] = crc;
+        h[6] = static_cast<uint32_t>(cd.tensor_off);
+        h[7] = static_cast<uint32_t>(cd.tensor_off >> 32);
+        h[8] = static_cast<uint32_t>(cd.len);
+        h[9] = static_cast<uint32_t>(cd.len >> 32);
+        h[10] = static_cast<uint32_t>(cd.payload_off);
+        h[11] = static_cast<uint32_t>(cd.payload_off >> 32);
+        h[12] = static_cast<uint32_t>(sbits);
+        h[13] = static_cast<uint32_t>(sbits >> 32);
+        h[14] = nonfinite;
+        uint32_t r = 0xFFFFFFFFu;
+        for (int i = 0; i < 15; ++i)
+          for (int j = 0; j < 4; ++j) r = crc_byte(T, r, (h[i] >> (8 * j)) & 0xFFu);
+        h[15] = r ^ 0xFFFFFFFFu;
+        uint4* dst = reinterpret_cast<uint4*>(p.packed + c * kHeaderBytes);
+        for (int q = 0; q < 4; ++q) dst[q] = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+      }
+      for (uint64_t j = pad_begin + lane; j < pad_end; j += 32) p.packed[j] = 0;
+      if (last)
+        for (uint64_t j = table_end + lane * 16u; j < gap_end; j += 512)
+          *reinterpret_cast<uint4*>(p.packed + j) = make_uint4(0, 0, 0, 0);
+    } else {  // unpack + verify
+      bool bad = false;
+      if (lane == 0) {
+        const uint4* src = reinterpret_cast<const uint4*>(p.packed + c * kHeaderBytes);
+        uint32_t h[16];
+        for (int q = 0; q < 4; ++q) {
+          const uint4 v = src[q];
+          h[4 * q] = v.x;
+          h[4 * q + 1] = v.y;
+          h[4 * q + 2] = v.z;
+          h[4 * q + 3] = v.w;
+        }
+        uint32_t r = 0xFFFFFFFFu;
+        for (int i = 0; i < 15; ++i)
+          for (int j = 0; j < 4; ++j) r = crc_byte(T, r, (h[i] >> (8 * j)) & 0xFFu);
+        bad = (h[15] != (r ^ 0xFFFFFFFFu)) || h[0] != kMagic || (h[1] & 0xFFFFu) != kVersion ||
+              (h[1] >> 16) != cd.dtype || h[2] != static_cast<uint32_t>(c) ||
+              h[3] != static_cast<uint32_t>(c >> 32) || h[4] != cd.tensor_idx ||
+              h[6] != static_cast<uint32_t>(cd.tensor_off) || h[7] != static_cast<uint32_t>(cd.tensor_off >> 32) ||
+              h[8] != static_cast<uint32_t>(cd.len) || h[9] != static_cast<uint32_t>(cd.len >> 32) ||
+              h[10] != static_cast<uint32_t>(cd.payload_off) ||
+              h[11] != static_cast<uint32_t>(cd.payload_off >> 32) || h[5] != crc;
+      }
+      for (uint64_t j = pad_begin + lane; j < pad_end; j += 32)
+        if (p.packed[j] != 0) bad = true;
+      if (last)
+        for (uint64_t j = table_end + lane; j < gap_end; j += 32)
+          if (p.packed[j] != 0) bad = true;
+      bad = __any_sync(kFull, bad);
+      if (lane == 0) p.flags[c] = bad ? 1 : 0;
+    }
+  }
+}
+
+// ------------------------------------------------------------------ compaction
+
+constexpr int kCompactThreads = 1024;
+constexpr int kPerThread = 8;
+constexpr int kTile = kCompactThreads * kPerThread;
+
+struct FlagPred {
+  const uint8_t* flags;
+  __device__ __forceinline__ bool operator()(uint64_t i) const { return flags[i] != 0; }
+};
+
+struct DiffPred {
+  const uint4* a;
+  const uint4* b;
+  __device__ __forceinline__ bool operator()(uint64_t i) const {
+    const uint4 x = a[i], y = b[i];
+    return ((x.x ^ y.x) | (x.y ^ y.y) | (x.z ^ y.z) | (x.w ^ y.w)) != 0u;
+  }
+};
+
+// One CTA walks the index space in tiles of kTile; thread t tests kPerThread
+// consecutive indices of the tile, a block-wide exclusive scan of the per-thread
+// counts gives each thread its output position, and the ids are written in
+// ascending order.  Deterministic: no atomics decide any position.
+template <class Pred>
+__global__ void __launch_bounds__(kCompactThreads) compact_kernel(Pred pred, uint64_t n, uint32_t* out,
+                                                                  uint64_t cap, uint64_t* count,
+                                                                  uint32_t* status) {
+  __shared__ uint32_t warp_tot[kCompactThreads / 32];
+  __shared__ uint64_t base_sh;
+  const uint32_t tid = threadIdx.x, lane = tid & 31u, warp = tid >> 5;
+  uint64_t base = 0;
+  for (uint64_t t0 = 0; t0 < n; t0 += kTile) {
+    const uint64_t first = t0 + static_cast<uint64_t>(tid) * kPerThread;
+    uint32_t bits = 0;
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j)
+      if (first + j < n && pred(first + j)) bits |= 1u << j;
+    const uint32_t cnt = __popc(bits);
+    uint32_t inc = cnt;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const uint32_t v = __shfl_up_sync(kFull, inc, d);
+      if (lane >= static_cast<uint32_t>(d)) inc += v;
+    }
+    if (lane == 31) warp_tot[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+      uint32_t w = warp_tot[lane];
+      uint32_t winc = w;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const uint32_t v = __shfl_up_sync(kFull, winc, d);
+        if (lane >= static_cast<uint32_t>(d)) winc += v;
+      }
+      warp_tot[lane] = winc - w;  // exclusive prefix of warp totals
+      if (lane == 31) base_sh = base + winc;
+    }
+    __syncthreads();
+    uint64_t pos = base + warp_tot[warp] + (inc - cnt);
+    while (bits) {
+      const int j = __ffs(bits) - 1;
+      bits &= bits - 1;
+      if (pos < cap) out[pos] = static_cast<uint32_t>(first + j);
+      ++pos;
+    }
+    base = base_sh;
+    __syncthreads();
+  }
+  if (tid == 0) {
+    *count = base;
+    if (base > cap && status != nullptr) atomicOr(status, kStatusCapacity);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_finalize(int mode, const FinalizeParams& p, cudaStream_t s) {
+  if (p.n_chunks == 0) return cudaSuccess;
+  uint64_t want = (p.n_chunks + kFinWarps - 1) / kFinWarps;
+  const int grid = static_cast<int>(want < 4096 ? want : 4096);
+  if (mode == kModeFingerprint)
+    finalize_kernel<kModeFingerprint><<<grid, kFinThreads, 0, s>>>(p);
+  else if (mode == kModePack)
+    finalize_kernel<kModePack><<<grid, kFinThreads, 0, s>>>(p);
+  else
+    finalize_kernel<kModeUnpack><<<grid, kFinThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_compact_flags(const uint8_t* flags, uint64_t n, uint32_t* out, uint64_t cap,
+                                 uint64_t* count, uint32_t* status, cudaStream_t s) {
+  compact_kernel<FlagPred><<<1, kCompactThreads, 0, s>>>(FlagPred{flags}, n, out, cap, count, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_diff(const FpEntry* a, const FpEntry* b, uint64_t n, uint32_t* out, uint64_t cap,
+                        uint64_t* count, cudaStream_t s) {
+  DiffPred pred{reinterpret_cast<const uint4*>(a), reinterpret_cast<const uint4*>(b)};
+  compact_kernel<DiffPred><<<1, kCompactThreads, 0, s>>>(pred, n, out, cap, count, nullptr);
+  return cudaGetLastError();
+}
+
+}  // namespace frk

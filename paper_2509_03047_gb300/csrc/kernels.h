@@ -1,0 +1,57 @@
+// kernels.h -- launchers of the device kernels (internal to libflashrec).
+#pragma once
+
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+#include "layout.h"
+
+namespace frk {
+
+enum : int { kModeFingerprint = 0, kModePack = 1, kModeUnpack = 2 };
+
+struct SweepParams {
+  const ChunkDesc* chunks;
+  const WarpDesc* warps;  // this class's per-warp ranges
+  const uint32_t* class_chunks;  // ids of this class's chunks with a body, in order
+  Record* recs;
+  uint8_t* packed;        // pack: destination; unpack: source; fingerprint: unused
+  uint32_t n_warps;       // warps with a descriptor
+};
+
+struct FinalizeParams {
+  const ChunkDesc* chunks;
+  const Record* recs;
+  const uint64_t* rec_nblk;
+  uint64_t n_chunks;
+  uint8_t* packed;  // pack: destination; unpack: source
+  FpEntry* out_fp;  // fingerprint: output table
+  uint8_t* flags;   // unpack: per-chunk verdict
+};
+
+// Geometry of the sweep kernel: one CTA of kSweepWarps warps per SM.
+#ifndef FR_SWEEP_WARPS
+#define FR_SWEEP_WARPS 16
+#endif
+constexpr int kSweepWarps = FR_SWEEP_WARPS;
+
+// Per device, before the first launch: opt the sweep kernels in to their
+// shared-memory size.
+cudaError_t configure_sweep_fp();
+cudaError_t configure_sweep_pack();
+cudaError_t configure_sweep_unpack();
+
+// One class of chunks: element type and 16-byte alignment of its tensors.
+cudaError_t launch_sweep_fp(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
+cudaError_t launch_sweep_pack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
+cudaError_t launch_sweep_unpack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
+cudaError_t launch_finalize(int mode, const FinalizeParams& p, cudaStream_t s);
+// Ascending ids of the set flags, first `cap` of them, and the true count.
+cudaError_t launch_compact_flags(const uint8_t* flags, uint64_t n, uint32_t* out, uint64_t cap,
+                                 uint64_t* count, uint32_t* status, cudaStream_t s);
+// Ascending ids of the differing 16-byte entries, first `cap`, true count.
+cudaError_t launch_diff(const FpEntry* a, const FpEntry* b, uint64_t n, uint32_t* out, uint64_t cap,
+                        uint64_t* count, cudaStream_t s);
+
+}  // namespace frk

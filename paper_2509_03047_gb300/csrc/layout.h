@@ -1,0 +1,70 @@
+// layout.h -- plan tables shared by the host planner and the kernels.
+//
+// A plan splits every tensor into chunks (per tensor, chunk_bytes each, the
+// last one shorter).  Each chunk is a "body" of whole 512-byte blocks plus a
+// "tail" of len % 512 bytes.  Chunks fall into sweep classes by element type
+// and by whether their tensor is 16-byte aligned.  The bodies of a class's
+// chunks, concatenated in chunk order, form one block stream that is cut into
+// equal ranges, one per warp of that class's sweep kernel, so every warp moves
+// the same number of bytes whatever the tensor sizes.  A warp's range overlaps
+// one or more chunks; each overlap is a "piece" and produces one record (raw
+// CRC, non-finite count, sum of squares).
+// The records of a chunk are consecutive and in order.  The finalize kernel
+// (one warp per chunk) folds a chunk's records and its tail.
+#pragma once
+
+#include <cstdint>
+
+namespace frk {
+
+constexpr uint64_t kHeaderBytes = 64;
+constexpr uint64_t kPayloadAlign = 256;
+constexpr uint32_t kMagic = 0x31435246u;  // bytes 'F','R','C','1'
+constexpr uint32_t kVersion = 1;
+
+enum : uint32_t { kDtBytes = 0, kDtBf16 = 1, kDtF32 = 2 };
+
+struct ChunkDesc {       // 64 bytes
+  uint64_t addr;         // device address of the chunk's first byte in its tensor
+  uint64_t len;          // chunk bytes
+  uint64_t tensor_off;   // offset of the chunk inside its tensor
+  uint64_t payload_off;  // offset of the payload in the packed buffer
+  uint64_t blk_begin;    // first body block in its class's block stream
+  uint32_t tensor_idx;
+  uint32_t dtype;
+  uint32_t first_rec;    // records of this chunk: [first_rec, first_rec + n_recs)
+  uint32_t n_recs;
+  uint32_t sweep_class;  // dtype * 2 + (tensor 16-byte aligned ? 1 : 0)
+  uint32_t pad1;
+};
+static_assert(sizeof(ChunkDesc) == 64, "ChunkDesc layout");
+
+struct WarpDesc {        // 32 bytes
+  uint64_t blk_begin;    // first block of this warp's range
+  uint64_t nblk;         // blocks in the range (0: idle warp)
+  uint32_t first_chunk;  // position, in the class's chunk list, of the chunk holding blk_begin
+  uint32_t rec_base;     // record index of the first piece
+  uint64_t pad;
+};
+static_assert(sizeof(WarpDesc) == 32, "WarpDesc layout");
+
+struct Record {          // one piece's partial result
+  uint32_t crc;          // raw CRC (preset 0, no final XOR) of the piece's bytes
+  uint32_t nonfinite;
+  double sumsq;
+};
+static_assert(sizeof(Record) == 16, "Record layout");
+
+struct FpEntry {         // = fr_fp
+  uint32_t crc32c;
+  uint32_t nonfinite;
+  double sumsq;
+};
+static_assert(sizeof(FpEntry) == 16, "FpEntry layout");
+
+// Device-side status bits (plan scratch).
+enum : uint32_t { kStatusCapacity = 1u, kStatusTimeout = 2u };
+
+constexpr uint64_t align_up(uint64_t v, uint64_t a) { return (v + a - 1) / a * a; }
+
+}  // namespace frk

@@ -1,0 +1,497 @@
+// sweep_impl.cuh -- the bandwidth-bound body sweep of fingerprint / pack / unpack.
+//
+// Restoration of a rank's state from a data-parallel replica (FlashRecovery,
+// arXiv 2509.03047, Sec. III-E) is, on one GPU, a sweep over every byte of
+// the param / master / Adam-m / Adam-v tensors: checksum it, and for the
+// transfer copy it into (pack) or out of (unpack) a flat buffer.  This kernel
+// does the whole-512-byte-block part of every chunk in one HBM pass:
+//
+//  * copy engine: each lane moves 16 bytes per block with a coalesced 128-bit
+//    load and (pack/unpack) a coalesced 128-bit store;
+//  * CRC-32C: the 128 words of a block are 128 interleaved CRC streams
+//    (lane l owns streams 4l..4l+3, four independent dependency chains), each
+//    advanced by s <- (s ^ w) * x^4096 with four byte lookups in tables kept in
+//    shared memory.  Every lane has a private copy of each table entry in its
+//    own bank, so the 32 lookups of a warp never conflict.  At the end of a
+//    piece the streams are folded with GF(2) multiplications by constants and
+//    warp shuffles into the raw CRC of the piece;
+//  * non-finite count and sum of squares, fused on the same registers: exact
+//    squares (fp32: x*x and fma(x,x,-x*x); bf16: x*x is already exact) summed
+//    with error-free TwoSum in packed f32x2 arithmetic, flushed into fp64.  A
+//    stage whose running sum is not finite (NaN/Inf input, or overflow) or is
+//    tiny with non-zero input is discarded and redone element by element in
+//    fp64 from a reload of its 16-byte units, so the fast path never needs a
+//    per-element test.
+//
+// No tensor cores: nothing here is a contraction.  One CTA of 16 warps per SM
+// (the 128 KiB of lane-replicated tables fill most of shared memory).  The
+// plan sorts chunks into classes by element type and by whether the tensor
+// is 16-byte aligned; each class gets its own block stream, cut into equal
+// per-warp ranges, and its own kernel specialization, so every kernel holds a
+// single loop variant and its registers.  sweep_{fp,pack,unpack}.cu each
+// instantiate one mode.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "gf2.cuh"
+#include "kernels.h"
+#include "layout.h"
+
+namespace frk {
+
+namespace {
+
+constexpr int kWarps = kSweepWarps;
+constexpr int kThreads = kWarps * 32;
+constexpr int kTableBytes = 4 * 256 * 32 * 4;  // 4 tables x 256 entries x 32 lanes x 4 B
+#ifndef FR_SWEEP_STAGE
+#define FR_SWEEP_STAGE 4
+#endif
+#ifndef FR_SWEEP_SPAN
+#define FR_SWEEP_SPAN 16
+#endif
+// Blocks per lane held in registers (one stage ahead).
+constexpr int kStage = FR_SWEEP_STAGE;
+// Blocks per validity span (a power of two, a multiple of kStage).
+constexpr int kSpan = FR_SWEEP_SPAN;
+// Spans prefetched into L2 ahead of use.
+constexpr int kAhead = 2;
+// Spans per fp32 partial sum before the fp64 flush: at most 128 elements per
+// f32x2 lane (bf16 adds two per block) keeps the TwoSum error term below 2^-34.
+constexpr int kFoldSpans = 64 / kSpan;
+static_assert(kSpan % kStage == 0 && (kSpan & (kSpan - 1)) == 0, "span geometry");
+static_assert(kFoldSpans >= 1, "fold geometry");
+
+typedef unsigned long long u64;
+
+__device__ const ByteTables4 g_braid = make_mul_tables(kBraidMul);
+
+extern __shared__ __align__(16) uint8_t g_smem[];
+
+// ------------------------------------------------------------------ tables
+
+// Table k, entry i, lane l lives at byte
+//   (k >> 1) * 65536 + i * 256 + (k & 1) * 128 + l * 4,
+// i.e. bank l.  The address of (table k, byte k of x, this lane) is one
+// byte-permute: byte 0 = l*4, byte 1 = byte k of x.
+__device__ __forceinline__ void fill_tables() {
+  for (int q = threadIdx.x; q < kTableBytes / 16; q += kThreads) {
+    const int k = q >> 11, rem = q & 2047, i = rem >> 3, g = rem & 7;
+    const uint32_t v = g_braid.t[k][i];
+    const uint32_t off = (k >> 1) * 65536 + i * 256 + (k & 1) * 128 + g * 16;
+    *reinterpret_cast<uint4*>(g_smem + off) = make_uint4(v, v, v, v);
+  }
+}
+
+__device__ __forceinline__ uint32_t tab(uint32_t off) {
+  return *reinterpret_cast<const uint32_t*>(g_smem + off);
+}
+
+// (s ^ w) * x^4096 for this lane's stream, given x = s ^ w.
+__device__ __forceinline__ uint32_t braid_step(uint32_t x, uint32_t lb) {
+  const uint32_t t0 = tab(__byte_perm(x, lb, 0x5504));
+  const uint32_t t1 = tab(__byte_perm(x, lb, 0x5514) + 128);
+  const uint32_t t2 = tab(__byte_perm(x, lb, 0x5524) + 65536);
+  const uint32_t t3 = tab(__byte_perm(x, lb, 0x5534) + 65536 + 128);
+  return (t0 ^ t1) ^ (t2 ^ t3);
+}
+
+// a * K mod P for a compile-time K: XOR of K * x^k over the set bits of a.
+template <uint32_t K>
+__device__ __forceinline__ uint32_t mulk(uint32_t a) {
+  uint32_t r = 0, b = K;
+#pragma unroll
+  for (int k = 0; k < 32; ++k) {
+    r ^= b & static_cast<uint32_t>(static_cast<int32_t>(a << k) >> 31);
+    b = gf_mul_x(b);
+  }
+  return r;
+}
+
+// ------------------------------------------------------------------ memory
+
+template <int AL>
+__device__ __forceinline__ uint4 ld_unit(const uint8_t* p);
+
+template <>
+__device__ __forceinline__ uint4 ld_unit<16>(const uint8_t* p) {
+  uint4 v;
+  asm("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
+      : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+      : "l"(p));
+  return v;
+}
+
+template <>
+__device__ __forceinline__ uint4 ld_unit<4>(const uint8_t* p) {
+  const uint32_t* q = reinterpret_cast<const uint32_t*>(p);
+  return make_uint4(__ldg(q), __ldg(q + 1), __ldg(q + 2), __ldg(q + 3));
+}
+
+template <>
+__device__ __forceinline__ uint4 ld_unit<1>(const uint8_t* p) {
+  uint32_t w[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    w[j] = static_cast<uint32_t>(__ldg(p + 4 * j)) | (static_cast<uint32_t>(__ldg(p + 4 * j + 1)) << 8) |
+           (static_cast<uint32_t>(__ldg(p + 4 * j + 2)) << 16) |
+           (static_cast<uint32_t>(__ldg(p + 4 * j + 3)) << 24);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+template <int AL>
+__device__ __forceinline__ void st_unit(uint8_t* p, uint4 v);
+
+template <>
+__device__ __forceinline__ void st_unit<16>(uint8_t* p, uint4 v) {
+  asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
+               : "memory");
+}
+
+template <>
+__device__ __forceinline__ void st_unit<4>(uint8_t* p, uint4 v) {
+  uint32_t* q = reinterpret_cast<uint32_t*>(p);
+  __stcs(q, v.x);
+  __stcs(q + 1, v.y);
+  __stcs(q + 2, v.z);
+  __stcs(q + 3, v.w);
+}
+
+template <>
+__device__ __forceinline__ void st_unit<1>(uint8_t* p, uint4 v) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int j = 0; j < 16; ++j) p[j] = static_cast<uint8_t>(w[j >> 2] >> (8 * (j & 3)));
+}
+
+// ------------------------------------------------------------------ f32x2
+
+__device__ __forceinline__ u64 pk(uint32_t lo, uint32_t hi) {
+  u64 r;
+  asm("mov.b64 %0, {%1,%2};" : "=l"(r) : "r"(lo), "r"(hi));
+  return r;
+}
+__device__ __forceinline__ float lo_f(u64 v) { return __uint_as_float(static_cast<uint32_t>(v)); }
+__device__ __forceinline__ float hi_f(u64 v) { return __uint_as_float(static_cast<uint32_t>(v >> 32)); }
+__device__ __forceinline__ u64 add2(u64 a, u64 b) {
+  u64 r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ u64 sub2(u64 a, u64 b) {
+  u64 r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ u64 mul2(u64 a, u64 b) {
+  u64 r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+
+// S + C += p, error-free (Knuth's TwoSum): S takes the rounded sum, C the
+// rounding error.
+__device__ __forceinline__ void two_sum_acc(u64& S, u64& C, u64 p) {
+  const u64 t = add2(S, p);
+  const u64 z = sub2(t, S);
+  const u64 y = sub2(t, z);
+  const u64 a = sub2(S, y);
+  const u64 b = sub2(p, z);
+  C = add2(C, add2(a, b));
+  S = t;
+}
+
+struct FpAcc {
+  u64 A, CA, B, CB;  // two f32x2 accumulators with their error terms
+  uint32_t any;      // OR of the stage's raw words (zero test)
+};
+
+template <int DT>
+__device__ __forceinline__ void fp_unit(const uint4& v, FpAcc& f) {
+  if (DT == kDtF32) {
+    const u64 x01 = pk(v.x, v.y), x23 = pk(v.z, v.w);
+    const u64 p01 = mul2(x01, x01), p23 = mul2(x23, x23);
+    // x*x = p + e exactly (fp32 product, FMA residual)
+    const float e0 = __fmaf_rn(__uint_as_float(v.x), __uint_as_float(v.x), -lo_f(p01));
+    const float e1 = __fmaf_rn(__uint_as_float(v.y), __uint_as_float(v.y), -hi_f(p01));
+    const float e2 = __fmaf_rn(__uint_as_float(v.z), __uint_as_float(v.z), -lo_f(p23));
+    const float e3 = __fmaf_rn(__uint_as_float(v.w), __uint_as_float(v.w), -hi_f(p23));
+    two_sum_acc(f.A, f.CA, p01);
+    f.CA = add2(f.CA, pk(__float_as_uint(e0), __float_as_uint(e1)));
+    two_sum_acc(f.B, f.CB, p23);
+    f.CB = add2(f.CB, pk(__float_as_uint(e2), __float_as_uint(e3)));
+  } else {
+    // bf16 pairs: the low element is the low half-word
+    const u64 y0 = pk(v.x << 16, v.x & 0xFFFF0000u), y1 = pk(v.y << 16, v.y & 0xFFFF0000u);
+    const u64 y2 = pk(v.z << 16, v.z & 0xFFFF0000u), y3 = pk(v.w << 16, v.w & 0xFFFF0000u);
+    two_sum_acc(f.A, f.CA, mul2(y0, y0));
+    two_sum_acc(f.B, f.CB, mul2(y2, y2));
+    two_sum_acc(f.A, f.CA, mul2(y1, y1));
+    two_sum_acc(f.B, f.CB, mul2(y3, y3));
+  }
+  f.any |= (v.x | v.y) | (v.z | v.w);
+}
+
+// Exact per-element fallback for this lane's units of blocks [b0, b1).
+template <int DT, int AL>
+__device__ __noinline__ void slow_span(const uint8_t* sp, uint64_t b0, uint64_t b1, uint32_t& nonfinite,
+                                       double& d) {
+  for (uint64_t b = b0; b < b1; ++b) {
+    const uint4 v = ld_unit<AL>(sp + b * kBlockBytes);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    for (int j = 0; j < 4; ++j) {
+      if (DT == kDtF32) {
+        if ((w[j] & 0x7F800000u) == 0x7F800000u) {
+          ++nonfinite;
+        } else {
+          const double x = static_cast<double>(__uint_as_float(w[j]));
+          d = __dadd_rn(d, __dmul_rn(x, x));
+        }
+      } else {
+        for (int h = 0; h < 2; ++h) {
+          const uint32_t bits = (w[j] >> (16 * h)) & 0xFFFFu;
+          if ((bits & 0x7F80u) == 0x7F80u) {
+            ++nonfinite;
+          } else {
+            const double x = static_cast<double>(__uint_as_float(bits << 16));
+            d = __dadd_rn(d, __dmul_rn(x, x));
+          }
+        }
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ double fold_to_double(const FpAcc& f) {
+  return ((static_cast<double>(lo_f(f.A)) + static_cast<double>(hi_f(f.A))) +
+          (static_cast<double>(lo_f(f.B)) + static_cast<double>(hi_f(f.B)))) +
+         ((static_cast<double>(lo_f(f.CA)) + static_cast<double>(hi_f(f.CA))) +
+          (static_cast<double>(lo_f(f.CB)) + static_cast<double>(hi_f(f.CB))));
+}
+
+// ------------------------------------------------------------------ piece
+
+// Bulk prefetch of [p, p + bytes) into L2 (TMA unit; no registers held).
+__device__ __forceinline__ void prefetch_l2(const uint8_t* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+// One piece: `nblk` 512-byte blocks from `src` (to `dst` for pack/unpack).
+// SAL / DAL: alignment class (16, 4 or 1 bytes) of the source / destination.
+//
+// Pipeline: lane 0 prefetches whole spans (kSpan blocks) into L2 kAhead spans
+// ahead with the bulk-copy unit; each lane keeps kStage 16-byte units of the
+// next stage in flight in registers, which therefore only cover L2 latency.
+// Validity of the fast fp32 sums is checked once per span; a failing span is
+// rolled back to its snapshot and redone exactly from a reload.
+template <int MODE, int DT, int SAL, int DAL>
+__device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
+                                         uint64_t nblk, uint32_t lane, Record* rec) {
+  constexpr bool kFp = (MODE != kModeUnpack) && (DT != kDtBytes);
+  constexpr uint32_t kZeroMask = (DT == kDtF32) ? 0x7FFFFFFFu : 0x7FFF7FFFu;
+  const uint32_t lb = lane << 2;
+  const uint8_t* sp = src + lane * 16;
+  uint8_t* dp = dst + lane * 16;
+
+  if (SAL == 16 && lane == 0) {
+    const uint64_t first = nblk < kSpan * kAhead ? nblk : kSpan * kAhead;
+    prefetch_l2(src, static_cast<uint32_t>(first * kBlockBytes));
+  }
+
+  uint32_t s0 = 0, s1 = 0, s2 = 0, s3 = 0;
+  FpAcc f{0ull, 0ull, 0ull, 0ull, 0u};
+  FpAcc snap = f;
+  double d = 0.0;
+  uint32_t nonfinite = 0;
+  bool big = false;
+  int fold = 0;
+
+  uint4 cur[kStage];
+#pragma unroll
+  for (int u = 0; u < kStage; ++u)
+    if (u < nblk) cur[u] = ld_unit<SAL>(sp + static_cast<uint64_t>(u) * kBlockBytes);
+
+  for (uint64_t i = 0; i < nblk; i += kStage) {
+    if ((i & (kSpan - 1)) == 0) {
+      snap = f;
+      if (SAL == 16 && lane == 0) {
+        const uint64_t pf = i + kSpan * kAhead;
+        if (pf < nblk) {
+          const uint64_t n = (nblk - pf < kSpan) ? nblk - pf : kSpan;
+          prefetch_l2(src + pf * kBlockBytes, static_cast<uint32_t>(n * kBlockBytes));
+        }
+      }
+    }
+    if (i + kStage <= nblk) {
+#pragma unroll
+      for (int u = 0; u < kStage; ++u) {
+        const uint4 v = cur[u];
+        if (MODE != kModeFingerprint) st_unit<DAL>(dp + (i + u) * kBlockBytes, v);
+        s0 = braid_step(s0 ^ v.x, lb);
+        s1 = braid_step(s1 ^ v.y, lb);
+        s2 = braid_step(s2 ^ v.z, lb);
+        s3 = braid_step(s3 ^ v.w, lb);
+        if (kFp) fp_unit<DT>(v, f);
+        const uint64_t nx = i + kStage + u;
+        if (nx < nblk) cur[u] = ld_unit<SAL>(sp + nx * kBlockBytes);
+      }
+    } else {
+#pragma unroll
+      for (int u = 0; u < kStage; ++u) {
+        if (i + u < nblk) {
+          const uint4 v = cur[u];
+          if (MODE != kModeFingerprint) st_unit<DAL>(dp + (i + u) * kBlockBytes, v);
+          s0 = braid_step(s0 ^ v.x, lb);
+          s1 = braid_step(s1 ^ v.y, lb);
+          s2 = braid_step(s2 ^ v.z, lb);
+          s3 = braid_step(s3 ^ v.w, lb);
+          if (kFp) fp_unit<DT>(v, f);
+        }
+      }
+    }
+    const uint64_t nxt = i + kStage;
+    if (kFp && ((nxt & (kSpan - 1)) == 0 || nxt >= nblk)) {
+      const u64 ab = add2(f.A, f.B);
+      const float tot = lo_f(ab) + hi_f(ab);
+      const uint32_t anym = f.any & kZeroMask;
+      f.any = 0;
+      // Finite, and either large enough that fp32 underflow is negligible
+      // (below 2^-80 relative) or made of zeros only.
+      const bool ok = (tot < __int_as_float(0x7F800000)) && (tot >= 0x1p-60f || anym == 0u || big);
+      if (!ok) {
+        f = snap;
+        f.any = 0;
+        const uint64_t s_begin = i & ~static_cast<uint64_t>(kSpan - 1);
+        slow_span<DT, SAL>(sp, s_begin, (nxt < nblk ? nxt : nblk), nonfinite, d);
+      }
+      if (++fold == kFoldSpans) {
+        d += fold_to_double(f);
+        big = big || (d >= 0x1p-60);
+        f.A = f.CA = f.B = f.CB = 0ull;
+        fold = 0;
+      }
+    }
+  }
+
+  // ---- fold the 128 streams into the raw CRC of the piece
+  uint32_t v = mulk<gf_xpow(32)>(s0) ^ s1;
+  v = mulk<gf_xpow(32)>(v) ^ s2;
+  v = mulk<gf_xpow(32)>(v) ^ s3;
+  {
+    uint32_t o;
+    o = __shfl_down_sync(0xFFFFFFFFu, v, 1);
+    v = mulk<gf_xpow(128)>(v) ^ o;
+    o = __shfl_down_sync(0xFFFFFFFFu, v, 2);
+    v = mulk<gf_xpow(256)>(v) ^ o;
+    o = __shfl_down_sync(0xFFFFFFFFu, v, 4);
+    v = mulk<gf_xpow(512)>(v) ^ o;
+    o = __shfl_down_sync(0xFFFFFFFFu, v, 8);
+    v = mulk<gf_xpow(1024)>(v) ^ o;
+    o = __shfl_down_sync(0xFFFFFFFFu, v, 16);
+    v = mulk<gf_xpow(2048)>(v) ^ o;
+  }
+
+  if (kFp) {
+    d += fold_to_double(f);
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) {
+      d += __shfl_down_sync(0xFFFFFFFFu, d, m);
+      nonfinite += __shfl_down_sync(0xFFFFFFFFu, nonfinite, m);
+    }
+  }
+  if (lane == 0) {
+    Record r;
+    r.crc = mulk<kUnbraid>(v);
+    r.nonfinite = nonfinite;
+    r.sumsq = d;
+    *rec = r;
+  }
+}
+
+template <int MODE, int DT, int AL>
+__device__ __forceinline__ void sweep_piece_al(const uint8_t* tensor, uint8_t* packed, uint64_t n,
+                                               uint32_t lane, Record* rec) {
+  if (MODE == kModeUnpack)
+    sweep_piece<MODE, DT, 16, AL>(packed, const_cast<uint8_t*>(tensor), n, lane, rec);
+  else
+    sweep_piece<MODE, DT, AL, 16>(tensor, packed, n, lane, rec);
+}
+
+// One kernel per (mode, element type, alignment class).  ALIGNED: every
+// tensor of the class is 16-byte aligned (128-bit loads and stores); else the
+// tensor side uses 32-bit or byte accesses, chosen per piece.
+template <int MODE, int DT, bool ALIGNED>
+__global__ void __launch_bounds__(kThreads, 1) sweep_kernel(SweepParams p) {
+  fill_tables();
+  __syncthreads();
+  const uint32_t lane = threadIdx.x & 31u;
+  const uint32_t w = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (w >= p.n_warps) return;
+  const WarpDesc wd = p.warps[w];
+  uint64_t b = wd.blk_begin, left = wd.nblk;
+  uint32_t k = wd.first_chunk, r = wd.rec_base;
+  while (left > 0) {
+    const ChunkDesc cd = p.chunks[p.class_chunks[k]];
+    const uint64_t nb = cd.len / kBlockBytes;
+    const uint64_t off = b - cd.blk_begin;
+    const uint64_t n = (left < nb - off) ? left : nb - off;
+    const uint8_t* tensor = reinterpret_cast<const uint8_t*>(cd.addr) + off * kBlockBytes;
+    uint8_t* packed = (MODE == kModeFingerprint) ? nullptr : p.packed + cd.payload_off + off * kBlockBytes;
+    if (ALIGNED) {
+      sweep_piece_al<MODE, DT, 16>(tensor, packed, n, lane, p.recs + r);
+    } else if ((reinterpret_cast<uintptr_t>(tensor) & 3u) == 0) {
+      sweep_piece_al<MODE, DT, 4>(tensor, packed, n, lane, p.recs + r);
+    } else {
+      sweep_piece_al<MODE, DT, 1>(tensor, packed, n, lane, p.recs + r);
+    }
+    ++r;
+    b += n;
+    left -= n;
+    ++k;
+  }
+}
+
+template <int MODE, int DT, bool ALIGNED>
+cudaError_t configure_one() {
+  return cudaFuncSetAttribute(sweep_kernel<MODE, DT, ALIGNED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              kTableBytes);
+}
+
+template <int MODE, int DT, bool ALIGNED>
+cudaError_t launch_one(const SweepParams& p, int n_ctas, cudaStream_t s) {
+  sweep_kernel<MODE, DT, ALIGNED><<<n_ctas, kThreads, kTableBytes, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+// Configure / launch every class kernel of one mode (unpack ignores the
+// element type: it only checksums and copies).
+template <int MODE>
+cudaError_t configure_mode() {
+  cudaError_t e = configure_one<MODE, kDtBytes, true>();
+  if (e == cudaSuccess) e = configure_one<MODE, kDtBytes, false>();
+  if (MODE != kModeUnpack) {
+    if (e == cudaSuccess) e = configure_one<MODE, kDtBf16, true>();
+    if (e == cudaSuccess) e = configure_one<MODE, kDtBf16, false>();
+    if (e == cudaSuccess) e = configure_one<MODE, kDtF32, true>();
+    if (e == cudaSuccess) e = configure_one<MODE, kDtF32, false>();
+  }
+  return e;
+}
+
+template <int MODE>
+cudaError_t launch_mode(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s) {
+  if (MODE == kModeUnpack || dtype == kDtBytes)
+    return aligned ? launch_one<MODE, kDtBytes, true>(p, n_ctas, s) : launch_one<MODE, kDtBytes, false>(p, n_ctas, s);
+  if (dtype == kDtBf16)
+    return aligned ? launch_one<MODE, kDtBf16, true>(p, n_ctas, s) : launch_one<MODE, kDtBf16, false>(p, n_ctas, s);
+  return aligned ? launch_one<MODE, kDtF32, true>(p, n_ctas, s) : launch_one<MODE, kDtF32, false>(p, n_ctas, s);
+}
+
+}  // namespace frk

@@ -1,0 +1,12 @@
+// sweep_pack.cu -- the pack specializations of the body sweep (sweep_impl.cuh).
+#include "sweep_impl.cuh"
+
+namespace frk {
+
+cudaError_t configure_sweep_pack() { return configure_mode<kModePack>(); }
+
+cudaError_t launch_sweep_pack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s) {
+  return launch_mode<kModePack>(dtype, aligned, p, n_ctas, s);
+}
+
+}  // namespace frk

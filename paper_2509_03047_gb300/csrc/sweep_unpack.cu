@@ -1,0 +1,12 @@
+// sweep_unpack.cu -- the unpack specializations of the body sweep (sweep_impl.cuh).
+#include "sweep_impl.cuh"
+
+namespace frk {
+
+cudaError_t configure_sweep_unpack() { return configure_mode<kModeUnpack>(); }
+
+cudaError_t launch_sweep_unpack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s) {
+  return launch_mode<kModeUnpack>(dtype, aligned, p, n_ctas, s);
+}
+
+}  // namespace frk
