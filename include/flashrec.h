@@ -151,6 +151,38 @@ fr_status fr_unpack_verify(fr_plan plan, const void* src, uint64_t src_bytes,
 fr_status fr_diff(const fr_fp* a_dev, const fr_fp* b_dev, uint64_t n_chunks,
                   uint32_t* diverged_dev, uint64_t cap, uint64_t* n_out_dev, void* stream);
 
+/* ---------------------------------------------------------------- no allocation */
+
+/* The paper has no counterpart to this call; it serves callers that cannot
+ * allocate device memory.  A recovery agent living inside a training process
+ * often finds every byte of the GPU reserved by the framework's allocator for
+ * the model and optimizer state, and some callers may not call
+ * cudaMalloc/cudaFree at all (their implicit device synchronization, or their
+ * failure when memory is exhausted, would break the caller).  fr_plan_create
+ * allocates, so such callers use this instead.
+ *
+ * fr_fingerprint_static computes exactly what fr_plan_create + fr_fingerprint
+ * + fr_plan_destroy compute for the same tensors and chunk size, writing
+ * n_chunks fr_fp entries to `out_dev`, but allocates nothing: its plan tables
+ * and scratch live in one fixed array in the library's device memory (a few
+ * MiB, held by every GPU that loads the library until the process exits), and
+ * its host-side planning uses fixed static tables.
+ *   - Limit: at most FR_STATIC_MAX_CHUNKS chunks and GPUs of at most 160 SMs;
+ *     larger inputs return FR_ERR_INVALID_ARG before any device work.
+ *   - The first call on a device sets that device up (looks up the array's
+ *     device address and configures the kernels), so make that first call
+ *     before any stream capture.
+ *   - Every call, on every stream, shares the one array and rewrites all of
+ *     it that it uses; calls whose work overlaps on the GPU (calls on
+ *     different streams with no ordering between them) race and give wrong
+ *     results.  Host-side calls are serialized by a lock.
+ *   - The table upload is a copy from pageable host memory, so the call
+ *     returns only after the work already queued on `stream` has finished.
+ * Errors: FR_ERR_INVALID_ARG (also for sizes beyond the limit), FR_ERR_CUDA. */
+#define FR_STATIC_MAX_CHUNKS 16384
+fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes,
+                                fr_fp* out_dev, void* stream);
+
 /* ---------------------------------------------------------------- status */
 
 /* Synchronize `stream`, then return and clear the first condition the plan's

@@ -16,7 +16,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libflashrec.so")
-SOURCES = ["sweep_fp.cu", "sweep_pack.cu", "sweep_unpack.cu", "finalize.cu", "api.cu"]
+SOURCES = ["sweep_fp.cu", "sweep_pack.cu", "sweep_unpack.cu", "finalize.cu", "api.cu", "static_fingerprint.cu"]
 HEADERS = ["gf2.cuh", "layout.h", "kernels.h", "sweep_impl.cuh"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

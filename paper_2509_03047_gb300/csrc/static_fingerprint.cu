@@ -1,0 +1,228 @@
+// static_fingerprint.cu -- fr_fingerprint_static: the fingerprint call for
+// callers that cannot allocate device memory.
+//
+// Who needs it: a recovery agent that runs inside a training process whose
+// framework allocator has already reserved all of the GPU's memory for the
+// model and optimizer state, or any code that is not allowed to call
+// cudaMalloc/cudaFree (their implicit device synchronization or their
+// failure when memory is exhausted would break the caller).  fr_plan_create
+// allocates the plan's tables and scratch, so such callers cannot use it.
+//
+// This entry point plans on the host into fixed-size static host tables and
+// runs the same sweep and finalize kernels as fr_fingerprint, with every
+// device table and the per-piece scratch in one file-scope __device__ array
+// below.  Every GPU that loads the library holds that array (a few MiB) until
+// the process exits.  Nothing here calls cudaMalloc, cudaFree or any other
+// allocating routine.
+//
+// Sharing: all calls, on every stream, use the same array, and each call
+// rewrites every table it uses before its kernels run, so nothing carries
+// over from the previous call.  Calls whose kernels overlap on the GPU (calls
+// on different streams without ordering between them) race on the array and
+// give wrong results.  Host-side planning is serialized by a mutex.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/flashrec.h"
+#include "gf2.cuh"
+#include "kernels.h"
+#include "layout.h"
+
+using namespace frk;
+
+namespace {
+
+// Limits of the static variant.
+constexpr uint64_t kMaxChunks = FR_STATIC_MAX_CHUNKS;
+constexpr uint64_t kMaxWarpsPerClass = 160 * kSweepWarps;  // up to 160 SMs
+constexpr uint64_t kClasses = 6;
+constexpr uint64_t kMaxWarps = kClasses * kMaxWarpsPerClass;
+constexpr uint64_t kMaxRecs = kMaxWarps + kMaxChunks;
+
+// Byte offsets of the tables inside the static array (256-byte aligned).
+constexpr uint64_t kOffChunks = 0;
+constexpr uint64_t kOffLists = align_up(kOffChunks + kMaxChunks * sizeof(ChunkDesc), 256);
+constexpr uint64_t kOffWarps = align_up(kOffLists + kMaxChunks * sizeof(uint32_t), 256);
+constexpr uint64_t kOffRecNblk = align_up(kOffWarps + kMaxWarps * sizeof(WarpDesc), 256);
+constexpr uint64_t kOffRecs = align_up(kOffRecNblk + kMaxRecs * sizeof(uint64_t), 256);
+constexpr uint64_t kScratchBytes = align_up(kOffRecs + kMaxRecs * sizeof(Record), 256);
+static_assert(kScratchBytes < (8ull << 20), "the static scratch must stay modest");
+
+// The device-side scratch.  In host code this name is only a stand-in for the
+// symbol, never a device address: kernels get the address that
+// cudaGetSymbolAddress returns for the current device.
+static __device__ __align__(256) uint8_t g_static_scratch[kScratchBytes];
+
+// Host copies of the tables, staged here and copied into the scratch.
+struct HostTables {
+  ChunkDesc chunks[kMaxChunks];
+  uint32_t lists[kMaxChunks];
+  WarpDesc warps[kMaxWarps];
+  uint64_t rec_nblk[kMaxRecs];
+};
+HostTables g_host;
+std::mutex g_mu;
+
+// Per-device set-up: the scratch address and the sweep kernels' shared-memory
+// opt-in, done on the first call with that device current.
+constexpr int kMaxDevices = 64;
+uint8_t* g_dev_ptr[kMaxDevices] = {};
+
+uint64_t elem_bytes(uint32_t dt) { return dt == kDtF32 ? 4 : (dt == kDtBf16 ? 2 : 1); }
+
+// `what` documents the reason at the call site; the status is what returns.
+fr_status fail(fr_status s, const char* what) {
+  (void)what;
+  return s;
+}
+
+fr_status setup_device(int dev, uint8_t** out) {
+  if (dev < 0 || dev >= kMaxDevices) return fail(FR_ERR_INVALID_ARG, "device index out of range");
+  if (g_dev_ptr[dev] == nullptr) {
+    void* ptr = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&ptr, g_static_scratch);
+    if (e != cudaSuccess || ptr == nullptr) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+    e = configure_sweep_fp();
+    if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+    g_dev_ptr[dev] = static_cast<uint8_t*>(ptr);
+  }
+  *out = g_dev_ptr[dev];
+  return FR_OK;
+}
+
+}  // namespace
+
+extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes,
+                                           fr_fp* out_dev, void* stream) {
+  if (n_tensors > 0 && tensors == nullptr) return fail(FR_ERR_INVALID_ARG, "tensors is null");
+  if (chunk_bytes == 0 || chunk_bytes % 4 != 0) return fail(FR_ERR_INVALID_ARG, "chunk_bytes must be a positive multiple of 4");
+  uint64_t n_chunks = 0;
+  for (uint64_t t = 0; t < n_tensors; ++t) {
+    const fr_tensor& x = tensors[t];
+    if (x.dtype > FR_DT_F32 || x.flags != 0) return fail(FR_ERR_INVALID_ARG, "bad dtype or flags");
+    if (x.nbytes % elem_bytes(x.dtype) != 0) return fail(FR_ERR_INVALID_ARG, "nbytes is not a multiple of the element size");
+    if (x.nbytes > 0 && x.ptr == nullptr) return fail(FR_ERR_INVALID_ARG, "tensor pointer is null");
+    if (x.nbytes >= (1ull << 47)) return fail(FR_ERR_INVALID_ARG, "tensor too large");
+    n_chunks += (x.nbytes + chunk_bytes - 1) / chunk_bytes;
+    if (n_chunks > kMaxChunks) return fail(FR_ERR_INVALID_ARG, "more chunks than FR_STATIC_MAX_CHUNKS");
+  }
+  if (n_chunks == 0) return FR_OK;
+  if (out_dev == nullptr) return fail(FR_ERR_INVALID_ARG, "out_dev is null");
+
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+  int n_sm = 0;
+  e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+  const uint64_t W = static_cast<uint64_t>(n_sm) * kSweepWarps;
+  if (W > kMaxWarpsPerClass) return fail(FR_ERR_INVALID_ARG, "GPU has more SMs than the static tables hold");
+
+  std::lock_guard<std::mutex> lk(g_mu);
+  uint8_t* scratch = nullptr;
+  fr_status st = setup_device(dev, &scratch);
+  if (st != FR_OK) return st;
+
+  // ---- plan into the static host tables (same rules as fr_plan_create)
+  HostTables& h = g_host;
+  uint64_t payload = align_up(n_chunks * kHeaderBytes, kPayloadAlign);
+  uint64_t class_blocks[kClasses] = {0, 0, 0, 0, 0, 0};
+  uint64_t c = 0;
+  for (uint64_t t = 0; t < n_tensors; ++t) {
+    const bool aligned = (reinterpret_cast<uintptr_t>(tensors[t].ptr) % 16 == 0) && (chunk_bytes % 16 == 0);
+    const uint32_t cls = tensors[t].dtype * 2 + (aligned ? 1 : 0);
+    for (uint64_t off = 0; off < tensors[t].nbytes; off += chunk_bytes) {
+      ChunkDesc& d = h.chunks[c++];
+      std::memset(&d, 0, sizeof d);
+      d.len = std::min<uint64_t>(chunk_bytes, tensors[t].nbytes - off);
+      d.addr = reinterpret_cast<uint64_t>(tensors[t].ptr) + off;
+      d.tensor_off = off;
+      d.payload_off = payload;
+      d.blk_begin = class_blocks[cls];
+      d.tensor_idx = static_cast<uint32_t>(t);
+      d.dtype = tensors[t].dtype;
+      d.sweep_class = cls;
+      payload += align_up(d.len, kPayloadAlign);
+      class_blocks[cls] += d.len / kBlockBytes;
+    }
+  }
+  struct Launch {
+    uint32_t dtype;
+    bool aligned;
+    uint64_t warp_off, list_off;
+  } launches[kClasses];
+  int n_launch = 0;
+  uint64_t n_warps = 0, n_lists = 0, n_recs = 0;
+  for (uint32_t cls = 0; cls < kClasses; ++cls) {
+    const uint64_t blk = class_blocks[cls];
+    if (blk == 0) continue;
+    Launch L{cls / 2, (cls & 1u) != 0, n_warps, n_lists};
+    for (uint64_t i = 0; i < n_chunks; ++i)
+      if (h.chunks[i].sweep_class == cls && h.chunks[i].len >= static_cast<uint64_t>(kBlockBytes))
+        h.lists[n_lists++] = static_cast<uint32_t>(i);
+    const uint32_t* list = h.lists + L.list_off;
+    uint64_t k = 0;
+    for (uint64_t w = 0; w < W; ++w) {
+      const uint64_t b0 = blk * w / W, b1 = blk * (w + 1) / W;
+      WarpDesc& wd = h.warps[n_warps++];
+      std::memset(&wd, 0, sizeof wd);
+      wd.blk_begin = b0;
+      wd.nblk = b1 - b0;
+      wd.rec_base = static_cast<uint32_t>(n_recs);
+      if (b1 == b0) continue;
+      while (b0 >= h.chunks[list[k]].blk_begin + h.chunks[list[k]].len / kBlockBytes) ++k;
+      wd.first_chunk = static_cast<uint32_t>(k);
+      uint64_t b = b0, j = k;
+      while (b < b1) {
+        ChunkDesc& d = h.chunks[list[j]];
+        const uint64_t end = d.blk_begin + d.len / kBlockBytes;
+        const uint64_t n = std::min(b1, end) - b;
+        if (d.n_recs == 0) d.first_rec = static_cast<uint32_t>(n_recs);
+        d.n_recs += 1;
+        h.rec_nblk[n_recs++] = n;  // n_recs <= W per class + chunks <= kMaxRecs
+        b += n;
+        if (b == end) ++j;
+      }
+    }
+    launches[n_launch++] = L;
+  }
+
+  // ---- tables into the scratch, ordered on the caller's stream
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  e = cudaMemcpyAsync(scratch + kOffChunks, h.chunks, n_chunks * sizeof(ChunkDesc), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess && n_lists)
+    e = cudaMemcpyAsync(scratch + kOffLists, h.lists, n_lists * sizeof(uint32_t), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess && n_warps)
+    e = cudaMemcpyAsync(scratch + kOffWarps, h.warps, n_warps * sizeof(WarpDesc), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess && n_recs)
+    e = cudaMemcpyAsync(scratch + kOffRecNblk, h.rec_nblk, n_recs * sizeof(uint64_t), cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+
+  const ChunkDesc* d_chunks = reinterpret_cast<const ChunkDesc*>(scratch + kOffChunks);
+  Record* d_recs = reinterpret_cast<Record*>(scratch + kOffRecs);
+  for (int i = 0; i < n_launch; ++i) {
+    SweepParams sp;
+    sp.chunks = d_chunks;
+    sp.warps = reinterpret_cast<const WarpDesc*>(scratch + kOffWarps) + launches[i].warp_off;
+    sp.class_chunks = reinterpret_cast<const uint32_t*>(scratch + kOffLists) + launches[i].list_off;
+    sp.recs = d_recs;
+    sp.packed = nullptr;
+    sp.n_warps = static_cast<uint32_t>(W);
+    e = launch_sweep_fp(launches[i].dtype, launches[i].aligned, sp, n_sm, s);
+    if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+  }
+  FinalizeParams fp;
+  fp.chunks = d_chunks;
+  fp.recs = d_recs;
+  fp.rec_nblk = reinterpret_cast<const uint64_t*>(scratch + kOffRecNblk);
+  fp.n_chunks = n_chunks;
+  fp.packed = nullptr;
+  fp.out_fp = reinterpret_cast<FpEntry*>(out_dev);
+  fp.flags = nullptr;
+  e = launch_finalize(kModeFingerprint, fp, s);
+  if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+  return FR_OK;
+}

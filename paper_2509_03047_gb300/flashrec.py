@@ -59,13 +59,14 @@ def _load() -> ctypes.CDLL:
     L.fr_unpack_verify.argtypes = [vp, vp, u64, vp, u64, vp, vp]
     L.fr_diff.argtypes = [vp, vp, u64, vp, u64, vp, vp]
     L.fr_sync_status.argtypes = [vp, vp]
+    L.fr_fingerprint_static.argtypes = [ctypes.POINTER(fr_tensor), u64, u64, vp, vp]
     L.fr_status_str.argtypes = [ctypes.c_int]
     L.fr_status_str.restype = ctypes.c_char_p
     L.fr_last_error.argtypes = []
     L.fr_last_error.restype = ctypes.c_char_p
     L.fr_version.argtypes = []
     for name in ["fr_plan_create", "fr_plan_info", "fr_plan_chunk", "fr_fingerprint", "fr_pack",
-                 "fr_unpack_verify", "fr_diff", "fr_sync_status", "fr_version"]:
+                 "fr_unpack_verify", "fr_diff", "fr_sync_status", "fr_version", "fr_fingerprint_static"]:
         getattr(L, name).restype = ctypes.c_int
     return L
 
@@ -172,6 +173,26 @@ def fr_diff(a: torch.Tensor, b: torch.Tensor, n_chunks: int, diverged: Optional[
 
 def fr_sync_status(plan, stream=None) -> int:
     return lib.fr_sync_status(plan, _stream(stream))
+
+
+FR_STATIC_MAX_CHUNKS = 16384
+
+
+def fr_fingerprint_static(tensors: Sequence[torch.Tensor], chunk_bytes: int, out: torch.Tensor,
+                          stream=None) -> None:
+    """The fingerprint without a plan and without any device allocation, for
+    callers that cannot allocate (see include/flashrec.h); `out` holds
+    n_chunks * 16 bytes."""
+    arr = (fr_tensor * max(1, len(tensors)))()
+    for i, t in enumerate(tensors):
+        if not t.is_contiguous():
+            raise ValueError("tensor %d is not contiguous" % i)
+        arr[i].ptr = t.data_ptr() if t.numel() else 0
+        arr[i].nbytes = t.numel() * t.element_size()
+        arr[i].dtype = fr_dtype_of(t)
+        arr[i].flags = 0
+    _check(lib.fr_fingerprint_static(arr, len(tensors), chunk_bytes, out.data_ptr() if out.numel() else None,
+                                     _stream(stream)), "fr_fingerprint_static")
 
 
 # ---------------------------------------------------------------- convenience
