@@ -72,44 +72,54 @@ def build(force: bool = False) -> str:
     return _SO
 
 
+def use_library(path=None) -> None:
+    """Load the oracle from another compiled copy (None: the default build).
+    Tests use this to run the pins against deliberately broken copies."""
+    global _LIB
+    _LIB = None
+    if path is not None:
+        _LIB = _bind(ctypes.CDLL(path))
+
+
 def lib() -> ctypes.CDLL:
     global _LIB
     if _LIB is None:
         build()
-        L = ctypes.CDLL(_SO)
-        u8p, u32p, u64p = (ctypes.POINTER(ctypes.c_uint8), ctypes.POINTER(ctypes.c_uint32),
-                           ctypes.POINTER(ctypes.c_uint64))
-        c_u32, c_u64 = ctypes.c_uint32, ctypes.c_uint64
-        L.or_crc_bitwise.argtypes = [c_u32, c_u32, c_u32, ctypes.c_void_p, c_u64]
-        L.or_crc_bitwise.restype = c_u32
-        L.or_crc_table.argtypes = [c_u32, c_u32, c_u32, ctypes.c_void_p, c_u64]
-        L.or_crc_table.restype = c_u32
-        L.or_crc_combine.argtypes = [c_u32, c_u32, c_u32, c_u64]
-        L.or_crc_combine.restype = c_u32
-        L.or_crc32c.argtypes = [ctypes.c_void_p, c_u64]
-        L.or_crc32c.restype = c_u32
-        L.or_crc32c_combine.argtypes = [c_u32, c_u32, c_u64]
-        L.or_crc32c_combine.restype = c_u32
-        L.or_fp_values.argtypes = [ctypes.c_void_p, c_u64, c_u32, u32p, ctypes.POINTER(ctypes.c_double)]
-        L.or_fp_values.restype = None
-        L.or_fingerprint_chunk.argtypes = [ctypes.c_void_p, c_u64, c_u32, ctypes.POINTER(_OrFp)]
-        L.or_fingerprint_chunk.restype = None
-        L.or_plan.argtypes = [u64p, u32p, c_u64, c_u64, ctypes.c_void_p, c_u64, u64p]
-        L.or_plan.restype = c_u64
-        L.or_header.argtypes = [ctypes.POINTER(_OrChunk), c_u64, ctypes.POINTER(_OrFp), ctypes.c_void_p]
-        L.or_header.restype = None
-        L.or_fingerprint.argtypes = [ctypes.POINTER(ctypes.c_void_p), u64p, u32p, c_u64, c_u64, ctypes.c_void_p]
-        L.or_fingerprint.restype = ctypes.c_int
-        L.or_pack.argtypes = [ctypes.POINTER(ctypes.c_void_p), u64p, u32p, c_u64, c_u64, ctypes.c_void_p, c_u64]
-        L.or_pack.restype = ctypes.c_int
-        L.or_unpack_verify.argtypes = [ctypes.POINTER(ctypes.c_void_p), u64p, u32p, c_u64, c_u64,
-                                       ctypes.c_void_p, c_u64, u32p, c_u64, u64p]
-        L.or_unpack_verify.restype = ctypes.c_int
-        L.or_diff.argtypes = [ctypes.c_void_p, ctypes.c_void_p, c_u64, u32p, c_u64]
-        L.or_diff.restype = c_u64
-        _ = (u8p,)
-        _LIB = L
+        _LIB = _bind(ctypes.CDLL(_SO))
     return _LIB
+
+
+def _bind(L: ctypes.CDLL) -> ctypes.CDLL:
+    u32p, u64p = ctypes.POINTER(ctypes.c_uint32), ctypes.POINTER(ctypes.c_uint64)
+    c_u32, c_u64 = ctypes.c_uint32, ctypes.c_uint64
+    L.or_crc_bitwise.argtypes = [c_u32, c_u32, c_u32, ctypes.c_void_p, c_u64]
+    L.or_crc_bitwise.restype = c_u32
+    L.or_crc_table.argtypes = [c_u32, c_u32, c_u32, ctypes.c_void_p, c_u64]
+    L.or_crc_table.restype = c_u32
+    L.or_crc_combine.argtypes = [c_u32, c_u32, c_u32, c_u64]
+    L.or_crc_combine.restype = c_u32
+    L.or_crc32c.argtypes = [ctypes.c_void_p, c_u64]
+    L.or_crc32c.restype = c_u32
+    L.or_crc32c_combine.argtypes = [c_u32, c_u32, c_u64]
+    L.or_crc32c_combine.restype = c_u32
+    L.or_fp_values.argtypes = [ctypes.c_void_p, c_u64, c_u32, u32p, ctypes.POINTER(ctypes.c_double)]
+    L.or_fp_values.restype = None
+    L.or_fingerprint_chunk.argtypes = [ctypes.c_void_p, c_u64, c_u32, ctypes.POINTER(_OrFp)]
+    L.or_fingerprint_chunk.restype = None
+    L.or_plan.argtypes = [u64p, u32p, c_u64, c_u64, ctypes.c_void_p, c_u64, u64p]
+    L.or_plan.restype = c_u64
+    L.or_header.argtypes = [ctypes.POINTER(_OrChunk), c_u64, ctypes.POINTER(_OrFp), ctypes.c_void_p]
+    L.or_header.restype = None
+    L.or_fingerprint.argtypes = [ctypes.POINTER(ctypes.c_void_p), u64p, u32p, c_u64, c_u64, ctypes.c_void_p]
+    L.or_fingerprint.restype = ctypes.c_int
+    L.or_pack.argtypes = [ctypes.POINTER(ctypes.c_void_p), u64p, u32p, c_u64, c_u64, ctypes.c_void_p, c_u64]
+    L.or_pack.restype = ctypes.c_int
+    L.or_unpack_verify.argtypes = [ctypes.POINTER(ctypes.c_void_p), u64p, u32p, c_u64, c_u64,
+                                   ctypes.c_void_p, c_u64, u32p, c_u64, u64p]
+    L.or_unpack_verify.restype = ctypes.c_int
+    L.or_diff.argtypes = [ctypes.c_void_p, ctypes.c_void_p, c_u64, u32p, c_u64]
+    L.or_diff.restype = c_u64
+    return L
 
 
 # ---------------------------------------------------------------- helpers

@@ -47,23 +47,31 @@ namespace {
 constexpr int kWarps = kSweepWarps;
 constexpr int kThreads = kWarps * 32;
 constexpr int kTableBytes = 4 * 256 * 32 * 4;  // 4 tables x 256 entries x 32 lanes x 4 B
-#ifndef FR_SWEEP_STAGE
-#define FR_SWEEP_STAGE 4
+// Pipeline geometry (compile-time; tuned on GB300 per mode).
+#ifndef FR_STAGE_FP
+#define FR_STAGE_FP 4
+#endif
+#ifndef FR_STAGE_PACK
+#define FR_STAGE_PACK 4
+#endif
+#ifndef FR_STAGE_UNPACK
+#define FR_STAGE_UNPACK 4
+#endif
+#ifndef FR_AHEAD_FP
+#define FR_AHEAD_FP 2
+#endif
+#ifndef FR_AHEAD_PACK
+#define FR_AHEAD_PACK 2
+#endif
+#ifndef FR_AHEAD_UNPACK
+#define FR_AHEAD_UNPACK 2
 #endif
 #ifndef FR_SWEEP_SPAN
 #define FR_SWEEP_SPAN 16
 #endif
-// Blocks per lane held in registers (one stage ahead).
-constexpr int kStage = FR_SWEEP_STAGE;
-// Blocks per validity span (a power of two, a multiple of kStage).
+// Blocks per validity span (a power of two, a multiple of every stage).
 constexpr int kSpan = FR_SWEEP_SPAN;
-// Spans prefetched into L2 ahead of use.
-constexpr int kAhead = 2;
-// Spans per fp32 partial sum before the fp64 flush: at most 128 elements per
-// f32x2 lane (bf16 adds two per block) keeps the TwoSum error term below 2^-34.
-constexpr int kFoldSpans = 64 / kSpan;
-static_assert(kSpan % kStage == 0 && (kSpan & (kSpan - 1)) == 0, "span geometry");
-static_assert(kFoldSpans >= 1, "fold geometry");
+static_assert((kSpan & (kSpan - 1)) == 0, "span geometry");
 
 typedef unsigned long long u64;
 
@@ -208,7 +216,6 @@ __device__ __forceinline__ void two_sum_acc(u64& S, u64& C, u64 p) {
 
 struct FpAcc {
   u64 A, CA, B, CB;  // two f32x2 accumulators with their error terms
-  uint32_t any;      // OR of the stage's raw words (zero test)
 };
 
 template <int DT>
@@ -234,13 +241,18 @@ __device__ __forceinline__ void fp_unit(const uint4& v, FpAcc& f) {
     two_sum_acc(f.A, f.CA, mul2(y1, y1));
     two_sum_acc(f.B, f.CB, mul2(y3, y3));
   }
-  f.any |= (v.x | v.y) | (v.z | v.w);
 }
+
+struct Exact {
+  double d;
+  uint32_t nonfinite;
+};
 
 // Exact per-element fallback for this lane's units of blocks [b0, b1).
 template <int DT, int AL>
-__device__ __noinline__ void slow_span(const uint8_t* sp, uint64_t b0, uint64_t b1, uint32_t& nonfinite,
-                                       double& d) {
+__device__ __noinline__ Exact slow_span(const uint8_t* sp, uint64_t b0, uint64_t b1) {
+  double d = 0.0;
+  uint32_t nonfinite = 0;
   for (uint64_t b = b0; b < b1; ++b) {
     const uint4 v = ld_unit<AL>(sp + b * kBlockBytes);
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
@@ -265,6 +277,19 @@ __device__ __noinline__ void slow_span(const uint8_t* sp, uint64_t b0, uint64_t 
       }
     }
   }
+  return Exact{d, nonfinite};
+}
+
+// Whether this lane's units of blocks [b0, b1) hold only (signed) zeros.
+template <int DT, int AL>
+__device__ __noinline__ bool span_is_zero(const uint8_t* sp, uint64_t b0, uint64_t b1) {
+  constexpr uint32_t kMask = (DT == kDtF32) ? 0x7FFFFFFFu : 0x7FFF7FFFu;
+  uint32_t acc = 0;
+  for (uint64_t b = b0; b < b1; ++b) {
+    const uint4 v = ld_unit<AL>(sp + b * kBlockBytes);
+    acc |= (v.x | v.y | v.z | v.w) & kMask;
+  }
+  return acc == 0;
 }
 
 __device__ __forceinline__ double fold_to_double(const FpAcc& f) {
@@ -281,45 +306,108 @@ __device__ __forceinline__ void prefetch_l2(const uint8_t* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
+// Per-mode pipeline geometry: blocks per lane held in registers one stage
+// ahead, and spans (kSpan blocks) prefetched into L2 ahead of use.
+template <int MODE>
+struct Geo {
+  static constexpr int kStage = MODE == kModeFingerprint ? FR_STAGE_FP : (MODE == kModePack ? FR_STAGE_PACK
+                                                                                              : FR_STAGE_UNPACK);
+  static constexpr int kAhead = MODE == kModeFingerprint ? FR_AHEAD_FP : (MODE == kModePack ? FR_AHEAD_PACK
+                                                                                              : FR_AHEAD_UNPACK);
+  static_assert(kSpan % kStage == 0, "a span holds whole stages");
+};
+
+// State of one lane while it sweeps a piece.
+template <int MODE, int DT>
+struct Lane {
+  uint32_t s[4];   // CRC streams 4l..4l+3
+  FpAcc f, snap;   // running fp32 sums and their value at the span start
+  double d;        // flushed sums
+  uint32_t nonfinite;
+  bool big;        // d already holds a sum >= 2^-60
+  int fold;
+};
+
+template <int MODE, int DT, int DAL>
+__device__ __forceinline__ void do_unit(Lane<MODE, DT>& L, const uint4& v, uint8_t* wp, uint32_t lb) {
+  constexpr bool kFp = (MODE != kModeUnpack) && (DT != kDtBytes);
+  if (MODE != kModeFingerprint) st_unit<DAL>(wp, v);
+  L.s[0] = braid_step(L.s[0] ^ v.x, lb);
+  L.s[1] = braid_step(L.s[1] ^ v.y, lb);
+  L.s[2] = braid_step(L.s[2] ^ v.z, lb);
+  L.s[3] = braid_step(L.s[3] ^ v.w, lb);
+  if (kFp) fp_unit<DT>(v, L.f);
+}
+
+// End of a span [b0, b1): the fast sums are kept if finite and either large
+// enough that fp32 underflow is negligible (below 2^-80 relative) or made of
+// zeros only; otherwise the span is redone exactly from a reload.
+template <int MODE, int DT, int SAL>
+__device__ __forceinline__ void span_end(Lane<MODE, DT>& L, const uint8_t* sp, uint64_t b0, uint64_t b1) {
+  constexpr int kFoldSpans = (DT == kDtF32 ? 128 : 64) / kSpan;  // <= 128 terms per f32x2 lane
+  const u64 ab = add2(L.f.A, L.f.B);
+  const float tot = lo_f(ab) + hi_f(ab);
+  bool ok = tot < __int_as_float(0x7F800000);
+  if (ok && !(tot >= 0x1p-60f) && !L.big) ok = span_is_zero<DT, SAL>(sp, b0, b1);
+  if (!ok) {
+    L.f = L.snap;
+    const Exact x = slow_span<DT, SAL>(sp, b0, b1);
+    L.d += x.d;
+    L.nonfinite += x.nonfinite;
+  }
+  if (++L.fold == kFoldSpans) {
+    L.d += fold_to_double(L.f);
+    L.big = L.big || (L.d >= 0x1p-60);
+    L.f.A = L.f.CA = L.f.B = L.f.CB = 0ull;
+    L.fold = 0;
+  }
+}
+
 // One piece: `nblk` 512-byte blocks from `src` (to `dst` for pack/unpack).
 // SAL / DAL: alignment class (16, 4 or 1 bytes) of the source / destination.
 //
-// Pipeline: lane 0 prefetches whole spans (kSpan blocks) into L2 kAhead spans
-// ahead with the bulk-copy unit; each lane keeps kStage 16-byte units of the
-// next stage in flight in registers, which therefore only cover L2 latency.
-// Validity of the fast fp32 sums is checked once per span; a failing span is
-// rolled back to its snapshot and redone exactly from a reload.
+// Pipeline: lane 0 prefetches whole spans into L2 kAhead spans ahead with the
+// bulk-copy unit; each lane keeps kStage 16-byte units of the next stage in
+// flight in registers, which therefore mostly wait for L2.  The sums' validity
+// is checked once per span; a failing span is rolled back to its snapshot and
+// redone exactly from a reload.
 template <int MODE, int DT, int SAL, int DAL>
 __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
-                                         uint64_t nblk, uint32_t lane, Record* rec) {
+                                            uint64_t nblk, uint32_t lane, Record* rec) {
   constexpr bool kFp = (MODE != kModeUnpack) && (DT != kDtBytes);
-  constexpr uint32_t kZeroMask = (DT == kDtF32) ? 0x7FFFFFFFu : 0x7FFF7FFFu;
+  constexpr int kStage = Geo<MODE>::kStage;
+  constexpr int kAhead = Geo<MODE>::kAhead;
+  constexpr uint32_t kStageBytes = kStage * kBlockBytes;
   const uint32_t lb = lane << 2;
   const uint8_t* sp = src + lane * 16;
-  uint8_t* dp = dst + lane * 16;
+  uint8_t* wp = dst + lane * 16;
 
-  if (SAL == 16 && lane == 0) {
+  if (kAhead > 0 && SAL == 16 && lane == 0) {
     const uint64_t first = nblk < kSpan * kAhead ? nblk : kSpan * kAhead;
     prefetch_l2(src, static_cast<uint32_t>(first * kBlockBytes));
   }
 
-  uint32_t s0 = 0, s1 = 0, s2 = 0, s3 = 0;
-  FpAcc f{0ull, 0ull, 0ull, 0ull, 0u};
-  FpAcc snap = f;
-  double d = 0.0;
-  uint32_t nonfinite = 0;
-  bool big = false;
-  int fold = 0;
+  Lane<MODE, DT> L;
+  L.s[0] = L.s[1] = L.s[2] = L.s[3] = 0;
+  L.f = FpAcc{0ull, 0ull, 0ull, 0ull};
+  L.snap = L.f;
+  L.d = 0.0;
+  L.nonfinite = 0;
+  L.big = false;
+  L.fold = 0;
 
   uint4 cur[kStage];
 #pragma unroll
   for (int u = 0; u < kStage; ++u)
     if (u < nblk) cur[u] = ld_unit<SAL>(sp + static_cast<uint64_t>(u) * kBlockBytes);
+  const uint8_t* lp = sp + kStageBytes;  // the next stage's loads
 
-  for (uint64_t i = 0; i < nblk; i += kStage) {
+  uint64_t i = 0;
+  // Steady state: this stage and the next are whole, so no predicates.
+  for (; i + 2 * kStage <= nblk; i += kStage) {
     if ((i & (kSpan - 1)) == 0) {
-      snap = f;
-      if (SAL == 16 && lane == 0) {
+      if (kFp) L.snap = L.f;
+      if (kAhead > 0 && SAL == 16 && lane == 0) {
         const uint64_t pf = i + kSpan * kAhead;
         if (pf < nblk) {
           const uint64_t n = (nblk - pf < kSpan) ? nblk - pf : kSpan;
@@ -327,61 +415,38 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
         }
       }
     }
-    if (i + kStage <= nblk) {
 #pragma unroll
-      for (int u = 0; u < kStage; ++u) {
+    for (int u = 0; u < kStage; ++u) {
+      const uint4 v = cur[u];
+      cur[u] = ld_unit<SAL>(lp + u * kBlockBytes);
+      do_unit<MODE, DT, DAL>(L, v, wp + u * kBlockBytes, lb);
+    }
+    lp += kStageBytes;
+    wp += kStageBytes;
+    if (kFp && ((i + kStage) & (kSpan - 1)) == 0) span_end<MODE, DT, SAL>(L, sp, i + kStage - kSpan, i + kStage);
+  }
+  // Drain: the last one or two stages, the last possibly partial.
+  for (; i < nblk; i += kStage) {
+    if ((i & (kSpan - 1)) == 0 && kFp) L.snap = L.f;
+#pragma unroll
+    for (int u = 0; u < kStage; ++u) {
+      if (i + u < nblk) {
         const uint4 v = cur[u];
-        if (MODE != kModeFingerprint) st_unit<DAL>(dp + (i + u) * kBlockBytes, v);
-        s0 = braid_step(s0 ^ v.x, lb);
-        s1 = braid_step(s1 ^ v.y, lb);
-        s2 = braid_step(s2 ^ v.z, lb);
-        s3 = braid_step(s3 ^ v.w, lb);
-        if (kFp) fp_unit<DT>(v, f);
-        const uint64_t nx = i + kStage + u;
-        if (nx < nblk) cur[u] = ld_unit<SAL>(sp + nx * kBlockBytes);
-      }
-    } else {
-#pragma unroll
-      for (int u = 0; u < kStage; ++u) {
-        if (i + u < nblk) {
-          const uint4 v = cur[u];
-          if (MODE != kModeFingerprint) st_unit<DAL>(dp + (i + u) * kBlockBytes, v);
-          s0 = braid_step(s0 ^ v.x, lb);
-          s1 = braid_step(s1 ^ v.y, lb);
-          s2 = braid_step(s2 ^ v.z, lb);
-          s3 = braid_step(s3 ^ v.w, lb);
-          if (kFp) fp_unit<DT>(v, f);
-        }
+        if (i + kStage + u < nblk) cur[u] = ld_unit<SAL>(lp + u * kBlockBytes);
+        do_unit<MODE, DT, DAL>(L, v, wp + u * kBlockBytes, lb);
       }
     }
-    const uint64_t nxt = i + kStage;
-    if (kFp && ((nxt & (kSpan - 1)) == 0 || nxt >= nblk)) {
-      const u64 ab = add2(f.A, f.B);
-      const float tot = lo_f(ab) + hi_f(ab);
-      const uint32_t anym = f.any & kZeroMask;
-      f.any = 0;
-      // Finite, and either large enough that fp32 underflow is negligible
-      // (below 2^-80 relative) or made of zeros only.
-      const bool ok = (tot < __int_as_float(0x7F800000)) && (tot >= 0x1p-60f || anym == 0u || big);
-      if (!ok) {
-        f = snap;
-        f.any = 0;
-        const uint64_t s_begin = i & ~static_cast<uint64_t>(kSpan - 1);
-        slow_span<DT, SAL>(sp, s_begin, (nxt < nblk ? nxt : nblk), nonfinite, d);
-      }
-      if (++fold == kFoldSpans) {
-        d += fold_to_double(f);
-        big = big || (d >= 0x1p-60);
-        f.A = f.CA = f.B = f.CB = 0ull;
-        fold = 0;
-      }
-    }
+    lp += kStageBytes;
+    wp += kStageBytes;
+    const uint64_t end = (i + kStage < nblk) ? i + kStage : nblk;
+    if (kFp && ((end & (kSpan - 1)) == 0 || end == nblk))
+      span_end<MODE, DT, SAL>(L, sp, i & ~static_cast<uint64_t>(kSpan - 1), end);
   }
 
   // ---- fold the 128 streams into the raw CRC of the piece
-  uint32_t v = mulk<gf_xpow(32)>(s0) ^ s1;
-  v = mulk<gf_xpow(32)>(v) ^ s2;
-  v = mulk<gf_xpow(32)>(v) ^ s3;
+  uint32_t v = mulk<gf_xpow(32)>(L.s[0]) ^ L.s[1];
+  v = mulk<gf_xpow(32)>(v) ^ L.s[2];
+  v = mulk<gf_xpow(32)>(v) ^ L.s[3];
   {
     uint32_t o;
     o = __shfl_down_sync(0xFFFFFFFFu, v, 1);
@@ -396,8 +461,10 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
     v = mulk<gf_xpow(2048)>(v) ^ o;
   }
 
+  double d = L.d;
+  uint32_t nonfinite = L.nonfinite;
   if (kFp) {
-    d += fold_to_double(f);
+    d += fold_to_double(L.f);
 #pragma unroll
     for (int m = 16; m >= 1; m >>= 1) {
       d += __shfl_down_sync(0xFFFFFFFFu, d, m);

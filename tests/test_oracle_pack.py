@@ -250,3 +250,29 @@ def test_empty_state(orc):
     assert rc == 0 and n == 0
     z = np.zeros(0, dtype=np.uint8)
     assert orc.pack([z], [DT_F32], CHUNK).size == 0
+
+
+@pytest.mark.parametrize("field_off,width", [(0, 4), (4, 2), (6, 2), (8, 8), (16, 4), (24, 8), (32, 8), (40, 8)])
+def test_wrong_field_under_a_valid_header_crc(orc, field_off, width):
+    """A header whose CRC is intact but whose addressing field disagrees with
+    the receiver's plan (a replayed or misdirected header) is flagged."""
+    arrs, dts = adversarial_state(9)
+    buf = orc.pack(arrs, dts, CHUNK)
+    c = 3
+    h = bytearray(buf[64 * c: 64 * c + 64].tobytes())
+    v = int.from_bytes(h[field_off:field_off + width], "little") ^ 1
+    h[field_off:field_off + width] = v.to_bytes(width, "little")
+    h[60:64] = orc.crc32c(bytes(h[:60])).to_bytes(4, "little")
+    bad = buf.copy()
+    bad[64 * c: 64 * c + 64] = np.frombuffer(bytes(h), dtype=np.uint8)
+    rc, ids, n = orc.unpack_verify(_fresh_dst(arrs), dts, CHUNK, bad)
+    assert list(ids) == [c]
+
+
+def test_swapped_headers_are_flagged(orc):
+    arrs, dts = adversarial_state(10)
+    buf = orc.pack(arrs, dts, CHUNK)
+    bad = buf.copy()
+    bad[64 * 2: 64 * 3], bad[64 * 5: 64 * 6] = buf[64 * 5: 64 * 6], buf[64 * 2: 64 * 3]
+    rc, ids, n = orc.unpack_verify(_fresh_dst(arrs), dts, CHUNK, bad)
+    assert list(ids) == [2, 5]
