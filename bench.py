@@ -256,7 +256,7 @@ def run_flashrec(args):
             return int(nmis.item()), int(ndiv.item())
         return None
 
-    launches_per_step = (n_cls + 1) * 2 + (n_cls + 1) + (n_cls + 2) + 1
+    launches_per_step = (n_cls + 1) * 2 + (n_cls + 1) + (n_cls + 2) + 1  # sweeps + finalize + compaction + diff
 
     # correctness of the timed configuration: the injected flips are found
     for _ in range(args.warmup):
@@ -313,17 +313,47 @@ def run_flashrec(args):
     e2e = None
     if not args.no_e2e:
         host_buf = plan_s.new_packed(pinned=True)
-        step(buf=host_buf, sync_counts=True)
+        # (a) the pipelined restore: batches packed on the replica's stream and
+        # unpacked on the receiver's stream as soon as each is packed, so both
+        # directions of the host link work at once; one re-send round
+        bs = fr.Plan(src, cfg.chunk_bytes, n_batches=args.batches)
+        bd = fr.Plan(dst, cfg.chunk_bytes, n_batches=args.batches)
+        s_src, s_dst = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+
+        def restore_step():
+            fr.fr_fingerprint(bs.handle, tab_s, s_src)
+            fr.fr_restore(bs.handle, bd.handle, host_buf, 1, mism, nmis, s_src, s_dst)
+            fr.fr_fingerprint(bd.handle, tab_d, s_dst)
+            fr.fr_diff(tab_s, tab_d, C, div, ndiv, s_dst)
+            s_dst.synchronize()
+            return int(nmis.item()), int(ndiv.item())  # the step's result, read on the host
+
+        restore_step()
         barrier()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         for _ in range(args.e2e_steps):
-            step(buf=host_buf, sync_counts=True)  # D2H pack, H2D unpack, D2H counts
+            e2e_found = restore_step()
         torch.cuda.synchronize()
         t_e2e = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
+        # (b) for comparison: whole-buffer pack, then whole-buffer unpack
+        step(buf=host_buf, sync_counts=True)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            step(buf=host_buf, sync_counts=True)
+        torch.cuda.synchronize()
+        t_serial = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
         e2e = {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_e2e / 1e9, dev), 2), "unit": "GB/s",
                "h2d_bytes_per_step": P, "d2h_bytes_per_step": P + 16, "ms_per_step": round(t_e2e * 1e3, 2),
-               "transfer": "pinned host buffer over NVLink-C2C, written and read by the kernels"}
+               "transfer": "pinned host buffer over NVLink-C2C; fr_restore with %d batches, pack and unpack on "
+                           "two streams, 1 re-send round; no injected flips" % bs.n_batches,
+               "found": {"mismatching_chunks": e2e_found[0], "diverged_chunks": e2e_found[1]},
+               "serial": {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_serial / 1e9, dev), 2),
+                          "ms_per_step": round(t_serial * 1e3, 2),
+                          "how": "fr_pack to the host buffer, then fr_unpack_verify from it, with the flips"}}
+        bs.close()
+        bd.close()
         del host_buf
 
     cpu = None
@@ -450,6 +480,7 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["flashrec", "reference"], default="flashrec")
     ap.add_argument("--config", default=DEFAULT_CONFIG)
     ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--batches", type=int, default=16)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-gb", type=float, default=1.0)

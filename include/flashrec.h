@@ -151,6 +151,55 @@ fr_status fr_unpack_verify(fr_plan plan, const void* src, uint64_t src_bytes,
 fr_status fr_diff(const fr_fp* a_dev, const fr_fp* b_dev, uint64_t n_chunks,
                   uint32_t* diverged_dev, uint64_t cap, uint64_t* n_out_dev, void* stream);
 
+/* ---------------------------------------------------------------- streamed restore */
+
+/* The transfer of Sec. III-E end to end: a healthy replica's state reaches a
+ * restarted rank through a transfer buffer, typically pinned host memory
+ * reached over NVLink-C2C.  A whole-buffer fr_pack followed by
+ * fr_unpack_verify uses one direction of that link at a time; the calls below
+ * split the chunks into batches so the replica packs batch b+1 while the
+ * rank unpacks batch b, and re-send only the chunks that fail verification.
+ *
+ * fr_plan_create_batched is fr_plan_create plus a split of the chunks into
+ * `n_batches` consecutive batches of about equal bytes (at most one per
+ * chunk).  Batch calls run on half the SMs, so a pack on one stream and an
+ * unpack on another share the GPU.  Whole-state calls on a batched plan behave
+ * exactly as on a plain one.  fr_plan_batch reports the batch count and a
+ * batch's chunk range. */
+fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes,
+                                 uint32_t n_batches, fr_plan* out);
+fr_status fr_plan_batch(fr_plan plan, uint32_t batch, uint32_t* n_batches, uint64_t* first_chunk,
+                        uint64_t* n_chunks);
+
+/* fr_pack / fr_unpack_verify restricted to one batch: the same bytes of the
+ * same packed layout (headers, payloads and padding of the batch's chunks;
+ * the table gap with the batch that holds the last chunk).  An unpacked
+ * batch only records its verdicts; fr_unpack_collect then lists the failing
+ * chunks of the plan's latest verdicts, exactly as fr_unpack_verify does. */
+fr_status fr_pack_batch(fr_plan plan, uint32_t batch, void* dst, uint64_t dst_bytes, void* stream);
+fr_status fr_unpack_verify_batch(fr_plan plan, uint32_t batch, const void* src, uint64_t src_bytes,
+                                 void* stream);
+fr_status fr_unpack_collect(fr_plan plan, uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev,
+                            void* stream);
+
+/* Re-send every chunk whose latest verdict in `dst` failed: re-pack it from
+ * `src` into `staging` on `stream_src`, then re-unpack and re-verify it on
+ * `stream_dst`.  Synchronizes `stream_dst` once to learn how many chunks fail
+ * (*n_resent, may be NULL).  `src` and `dst` must describe the same layout
+ * (else FR_ERR_PLAN_MISMATCH). */
+fr_status fr_resend(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint64_t* n_resent,
+                    void* stream_src, void* stream_dst);
+
+/* The whole restoration: for every batch, pack it from `src` on `stream_src`
+ * and, as soon as it is packed, unpack and verify it into `dst` on
+ * `stream_dst`; then up to `max_retries` rounds of fr_resend (each
+ * synchronizes `stream_dst` once); then list the chunks that still fail, as
+ * fr_unpack_verify does.  All work is ordered before later work on
+ * `stream_dst`.  With max_retries = 0 nothing synchronizes. */
+fr_status fr_restore(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint32_t max_retries,
+                     uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev, void* stream_src,
+                     void* stream_dst);
+
 /* ---------------------------------------------------------------- no allocation */
 
 /* The paper has no counterpart to this call; it serves callers that cannot
@@ -167,8 +216,10 @@ fr_status fr_diff(const fr_fp* a_dev, const fr_fp* b_dev, uint64_t n_chunks,
  * and scratch live in one fixed array in the library's device memory (a few
  * MiB, held by every GPU that loads the library until the process exits), and
  * its host-side planning uses fixed static tables.
- *   - Limit: at most FR_STATIC_MAX_CHUNKS chunks and GPUs of at most 160 SMs;
- *     larger inputs return FR_ERR_INVALID_ARG before any device work.
+ *   - Limits: at most FR_STATIC_MAX_CHUNKS chunks, at most
+ *     FR_STATIC_MAX_SEGMENTS 16 KiB segments of chunk bodies (2 GiB of state
+ *     in large chunks), and GPUs of at most 160 SMs; larger inputs return
+ *     FR_ERR_INVALID_ARG before any device work.
  *   - The first call on a device sets that device up (looks up the array's
  *     device address and configures the kernels), so make that first call
  *     before any stream capture.
@@ -180,6 +231,7 @@ fr_status fr_diff(const fr_fp* a_dev, const fr_fp* b_dev, uint64_t n_chunks,
  *     returns only after the work already queued on `stream` has finished.
  * Errors: FR_ERR_INVALID_ARG (also for sizes beyond the limit), FR_ERR_CUDA. */
 #define FR_STATIC_MAX_CHUNKS 16384
+#define FR_STATIC_MAX_SEGMENTS 131072
 fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes,
                                 fr_fp* out_dev, void* stream);
 

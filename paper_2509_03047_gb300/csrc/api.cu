@@ -2,9 +2,15 @@
 // host-side planner.
 //
 // The planner turns a tensor list into the device tables of layout.h:
-// per-tensor chunks, the packed layout, the equal per-warp block ranges of the
-// sweep and the record slots of every piece.  All device memory a plan needs is
-// allocated here, at creation; the four sweep calls only launch kernels.
+// per-tensor chunks, the packed layout, and one or two "decompositions" of the
+// chunk bodies into per-warp work.  The whole-state decomposition cuts each
+// (element type, alignment) class's block stream into equal ranges for the
+// warps of every SM; a batched plan also cuts the chunks into consecutive
+// batches of about equal bytes, each decomposed over half the SMs, so that a
+// replica's pack of batch b+1 and a restarted rank's unpack of batch b can run
+// side by side (a sweep CTA holds most of an SM's shared memory, so two
+// kernels only overlap on disjoint SMs).  All device memory and events a plan
+// needs are created here, at creation; the sweep calls only launch kernels.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -22,31 +28,53 @@
 
 using namespace frk;
 
-// One sweep class: chunks of one element type whose tensors are (or are not)
-// 16-byte aligned, with its own block stream and per-warp ranges.
+namespace {
+
+// One sweep class of one batch: its kernel specialization and its slices of
+// the decomposition's warp and chunk-list tables.
 struct SweepClass {
   uint32_t dtype = 0;
   bool aligned = false;
-  uint64_t n_blocks = 0;
-  uint64_t warp_off = 0;  // into d_warps
-  uint64_t list_off = 0;  // into d_class_chunks
+  uint64_t warp_off = 0;
+  uint64_t list_off = 0;
 };
+
+struct BatchInfo {
+  uint64_t c_begin = 0, c_end = 0;
+  std::vector<SweepClass> classes;
+};
+
+// Per-warp work of every batch, with the chunk table that carries this
+// decomposition's block offsets and record ranges.
+struct Decomp {
+  int n_ctas = 0;
+  uint32_t n_warps = 0;  // per class launch: n_ctas * kSweepWarps
+  std::vector<BatchInfo> batches;
+  uint64_t n_recs = 0;
+  ChunkDesc* d_chunks = nullptr;
+  WarpDesc* d_warps = nullptr;
+  uint32_t* d_lists = nullptr;
+  uint64_t* d_rec_nblk = nullptr;
+  Record* d_recs = nullptr;
+};
+
+}  // namespace
 
 struct fr_plan_s {
   int device = 0;
   int n_sm = 0;
   uint64_t chunk_bytes = 0, n_chunks = 0, packed_bytes = 0, state_bytes = 0;
-  uint64_t n_recs = 0;
-  uint32_t n_warps = 0;  // warps per class launch (n_sm * kSweepWarps)
-  std::vector<ChunkDesc> chunks;
-  std::vector<SweepClass> classes;  // non-empty classes, in class-id order
-  ChunkDesc* d_chunks = nullptr;
-  WarpDesc* d_warps = nullptr;
-  uint32_t* d_class_chunks = nullptr;
-  uint64_t* d_rec_nblk = nullptr;
-  Record* d_recs = nullptr;
-  uint8_t* d_flags = nullptr;
+  uint32_t n_batches = 1;
+  std::vector<ChunkDesc> chunks;  // layout fields (host copy)
+  Decomp whole;                   // one batch over all SMs
+  Decomp batched;                 // n_batches > 1: batches over half the SMs
+  uint64_t n_segs = 0;            // 16 KiB sum segments of all chunk bodies
+  double* d_segs = nullptr;       // their sums of squares
+  uint8_t* d_flags = nullptr;     // unpack verdict per chunk
   uint32_t* d_status = nullptr;
+  uint32_t* d_ids = nullptr;      // restore: ids of failing chunks (capacity n_chunks)
+  uint64_t* d_count = nullptr;
+  std::vector<cudaEvent_t> events;  // restore: one per batch, plus one
 };
 
 namespace {
@@ -113,14 +141,245 @@ cudaError_t upload(T** dst, const std::vector<T>& src) {
   return cudaMemcpy(*dst, src.data(), src.size() * sizeof(T), cudaMemcpyHostToDevice);
 }
 
+void free_decomp(Decomp& D) {
+  cudaFree(D.d_chunks);
+  cudaFree(D.d_warps);
+  cudaFree(D.d_lists);
+  cudaFree(D.d_rec_nblk);
+  cudaFree(D.d_recs);
+  D = Decomp();
+}
+
 void free_device(fr_plan p) {
-  cudaFree(p->d_chunks);
-  cudaFree(p->d_warps);
-  cudaFree(p->d_class_chunks);
-  cudaFree(p->d_rec_nblk);
-  cudaFree(p->d_recs);
+  free_decomp(p->whole);
+  free_decomp(p->batched);
+  cudaFree(p->d_segs);
   cudaFree(p->d_flags);
   cudaFree(p->d_status);
+  cudaFree(p->d_ids);
+  cudaFree(p->d_count);
+  for (cudaEvent_t ev : p->events) cudaEventDestroy(ev);
+  p->events.clear();
+}
+
+// Cut the chunks [bounds[b], bounds[b+1]) of every batch b into sweep work for
+// `n_ctas` CTAs: per batch and class, the class's 16 KiB segments in chunk
+// order are split into equal runs, one per warp, and every (warp, chunk)
+// overlap gets one record.  Records are numbered batch by batch, class
+// by class, so each chunk's records are consecutive.  `min_recs`: record slots
+// to allocate at least (list-mode calls use one slot per listed chunk).
+cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<uint64_t>& bounds, int n_ctas,
+                         uint64_t min_recs, Decomp& D) {
+  const uint64_t W = static_cast<uint64_t>(n_ctas) * kSweepWarps;
+  D.n_ctas = n_ctas;
+  D.n_warps = static_cast<uint32_t>(W);
+  std::vector<ChunkDesc> chunks = base;
+  std::vector<WarpDesc> warps;
+  std::vector<uint32_t> lists;
+  std::vector<uint64_t> rec_nblk;
+  for (ChunkDesc& d : chunks) {
+    d.blk_begin = 0;
+    d.first_rec = 0;
+    d.n_recs = 0;
+  }
+  for (size_t b = 0; b + 1 < bounds.size(); ++b) {
+    BatchInfo bi;
+    bi.c_begin = bounds[b];
+    bi.c_end = bounds[b + 1];
+    uint64_t class_blocks[6] = {0, 0, 0, 0, 0, 0};
+    for (uint64_t c = bi.c_begin; c < bi.c_end; ++c) {
+      ChunkDesc& d = chunks[c];
+      d.blk_begin = class_blocks[d.sweep_class];
+      class_blocks[d.sweep_class] += d.len / kBlockBytes;
+    }
+    for (uint32_t cls = 0; cls < 6; ++cls) {
+      const uint64_t blk = class_blocks[cls];
+      if (blk == 0) continue;
+      SweepClass sc;
+      sc.dtype = cls / 2;
+      sc.aligned = (cls & 1u) != 0;
+      sc.warp_off = warps.size();
+      sc.list_off = lists.size();
+      for (uint64_t c = bi.c_begin; c < bi.c_end; ++c)
+        if (chunks[c].sweep_class == cls && chunks[c].len >= static_cast<uint64_t>(kBlockBytes))
+          lists.push_back(static_cast<uint32_t>(c));
+      const size_t lbase = sc.list_off;
+      // warp ranges start on segment boundaries: cut the class's segments
+      // (not its blocks) evenly, then convert to block ranges
+      std::vector<uint64_t> seg_start;  // class-stream block where each segment starts
+      for (size_t q = lbase; q < lists.size(); ++q) {
+        const ChunkDesc& d = chunks[lists[q]];
+        const uint64_t nb = d.len / kBlockBytes;
+        for (uint64_t j = 0; j < nb; j += kSegBlocks) seg_start.push_back(d.blk_begin + j);
+      }
+      const uint64_t n_seg = seg_start.size();
+      seg_start.push_back(blk);
+      uint64_t k = 0;  // walks the class list monotonically
+      for (uint64_t w = 0; w < W; ++w) {
+        const uint64_t b0 = seg_start[n_seg * w / W], b1 = seg_start[n_seg * (w + 1) / W];
+        WarpDesc wd;
+        std::memset(&wd, 0, sizeof wd);
+        wd.blk_begin = b0;
+        wd.nblk = b1 - b0;
+        wd.rec_base = static_cast<uint32_t>(rec_nblk.size());
+        if (b1 > b0) {
+          while (b0 >= chunks[lists[lbase + k]].blk_begin + chunks[lists[lbase + k]].len / kBlockBytes) ++k;
+          wd.first_chunk = static_cast<uint32_t>(k);
+          uint64_t bb = b0, j = k;
+          while (bb < b1) {
+            ChunkDesc& d = chunks[lists[lbase + j]];
+            const uint64_t end = d.blk_begin + d.len / kBlockBytes;
+            const uint64_t n = std::min(b1, end) - bb;
+            if (d.n_recs == 0) d.first_rec = static_cast<uint32_t>(rec_nblk.size());
+            d.n_recs += 1;
+            rec_nblk.push_back(n);
+            bb += n;
+            if (bb == end) ++j;
+          }
+        }
+        warps.push_back(wd);
+      }
+      bi.classes.push_back(sc);
+    }
+    D.batches.push_back(bi);
+  }
+  D.n_recs = rec_nblk.size();
+  cudaError_t e = upload(&D.d_chunks, chunks);
+  if (e == cudaSuccess) e = upload(&D.d_warps, warps);
+  if (e == cudaSuccess) e = upload(&D.d_lists, lists);
+  if (e == cudaSuccess) e = upload(&D.d_rec_nblk, rec_nblk);
+  const uint64_t slots = std::max<uint64_t>(D.n_recs, min_recs);
+  if (e == cudaSuccess && slots) e = cudaMalloc(&D.d_recs, slots * sizeof(Record));
+  return e;
+}
+
+// Sweep + finalize of batches [b0, b1) of decomposition D.
+fr_status run_batches(fr_plan p, const Decomp& D, int mode, uint8_t* packed, FpEntry* out_fp, size_t b0, size_t b1,
+                      cudaStream_t s) {
+  for (size_t b = b0; b < b1; ++b) {
+    for (const SweepClass& sc : D.batches[b].classes) {
+      SweepParams sp;
+      sp.chunks = D.d_chunks;
+      sp.warps = D.d_warps + sc.warp_off;
+      sp.class_chunks = D.d_lists + sc.list_off;
+      sp.recs = D.d_recs;
+      sp.segs = p->d_segs;
+      sp.packed = packed;
+      sp.n_warps = D.n_warps;
+      cudaError_t e;
+      if (mode == kModeFingerprint)
+        e = launch_sweep_fp(sc.dtype, sc.aligned, sp, D.n_ctas, s);
+      else if (mode == kModePack)
+        e = launch_sweep_pack(sc.dtype, sc.aligned, sp, D.n_ctas, s);
+      else
+        e = launch_sweep_unpack(sc.dtype, sc.aligned, sp, D.n_ctas, s);
+      if (e != cudaSuccess) return cuda_fail(e, "sweep kernel launch");
+    }
+  }
+  FinalizeParams fp;
+  fp.chunks = D.d_chunks;
+  fp.recs = D.d_recs;
+  fp.segs = p->d_segs;
+  fp.rec_nblk = D.d_rec_nblk;
+  fp.n_chunks = p->n_chunks;
+  fp.c_begin = D.batches[b0].c_begin;
+  fp.c_end = D.batches[b1 - 1].c_end;
+  fp.ids = nullptr;
+  fp.packed = packed;
+  fp.out_fp = out_fp;
+  fp.flags = p->d_flags;
+  cudaError_t e = launch_finalize(mode, fp, s);
+  if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
+  return FR_OK;
+}
+
+// Sweep + finalize of the `n` chunks listed in `ids` (device), each by one
+// warp: used to re-send chunks that failed verification.
+fr_status run_list(fr_plan p, int mode, const uint32_t* ids, uint64_t n, uint8_t* packed, cudaStream_t s) {
+  if (n == 0) return FR_OK;
+  ListParams lp;
+  lp.chunks = p->whole.d_chunks;
+  lp.ids = ids;
+  lp.n = n;
+  lp.recs = p->whole.d_recs;
+  lp.segs = p->d_segs;
+  lp.packed = packed;
+  cudaError_t e = launch_list_sweep(mode, lp, s);
+  if (e != cudaSuccess) return cuda_fail(e, "list sweep kernel launch");
+  FinalizeParams fp;
+  fp.chunks = p->whole.d_chunks;
+  fp.recs = p->whole.d_recs;
+  fp.segs = p->d_segs;
+  fp.rec_nblk = nullptr;
+  fp.n_chunks = p->n_chunks;
+  fp.c_begin = 0;
+  fp.c_end = n;
+  fp.ids = ids;
+  fp.packed = packed;
+  fp.out_fp = nullptr;
+  fp.flags = p->d_flags;
+  e = launch_finalize(mode, fp, s);
+  if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
+  return FR_OK;
+}
+
+fr_status check_packed_buffer(fr_plan p, const void* buf, uint64_t bytes) {
+  if (buf == nullptr) return invalid("packed buffer is null");
+  if (reinterpret_cast<uintptr_t>(buf) % 16 != 0) {
+    set_err("packed buffer must be 16-byte aligned");
+    return FR_ERR_ALIGNMENT;
+  }
+  if (bytes < p->packed_bytes) {
+    set_err("packed buffer holds %llu bytes, plan needs %llu", (unsigned long long)bytes,
+            (unsigned long long)p->packed_bytes);
+    return FR_ERR_BUFFER_TOO_SMALL;
+  }
+  return FR_OK;
+}
+
+const Decomp& batch_decomp(fr_plan p) { return p->n_batches > 1 ? p->batched : p->whole; }
+
+fr_status check_same_layout(fr_plan src, fr_plan dst) {
+  if (src->device != dst->device || src->n_chunks != dst->n_chunks || src->packed_bytes != dst->packed_bytes ||
+      src->n_batches != dst->n_batches) {
+    set_err("the two plans do not describe the same layout");
+    return FR_ERR_PLAN_MISMATCH;
+  }
+  for (uint64_t c = 0; c < src->n_chunks; ++c) {
+    const ChunkDesc &a = src->chunks[c], &b = dst->chunks[c];
+    if (a.len != b.len || a.dtype != b.dtype || a.tensor_idx != b.tensor_idx || a.tensor_off != b.tensor_off) {
+      set_err("the two plans differ at chunk %llu", (unsigned long long)c);
+      return FR_ERR_PLAN_MISMATCH;
+    }
+  }
+  return FR_OK;
+}
+
+// One re-send: list the chunks whose last verdict in `dst` failed (a host
+// sync learns how many), re-pack them from `src` on `ss`, and re-unpack them
+// on `sd` after that.  *failing gets the number re-sent.
+fr_status resend_failed(fr_plan src, fr_plan dst, uint8_t* buf, cudaStream_t ss, cudaStream_t sd,
+                        uint64_t* failing) {
+  *failing = 0;
+  cudaError_t e =
+      launch_compact_flags(dst->d_flags, dst->n_chunks, dst->d_ids, dst->n_chunks, dst->d_count, nullptr, sd);
+  if (e != cudaSuccess) return cuda_fail(e, "compaction kernel launch");
+  uint64_t n = 0;
+  if ((e = cudaMemcpyAsync(&n, dst->d_count, sizeof n, cudaMemcpyDeviceToHost, sd)) != cudaSuccess ||
+      (e = cudaStreamSynchronize(sd)) != cudaSuccess)
+    return cuda_fail(e, "read failing-chunk count");
+  if (n == 0) return FR_OK;
+  cudaEvent_t ev_ids = dst->events[dst->n_batches], ev_packed = src->events[src->n_batches];
+  if ((e = cudaEventRecord(ev_ids, sd)) != cudaSuccess || (e = cudaStreamWaitEvent(ss, ev_ids, 0)) != cudaSuccess)
+    return cuda_fail(e, "order the re-send");
+  fr_status st = run_list(src, kModePack, dst->d_ids, n, buf, ss);
+  if (st != FR_OK) return st;
+  if ((e = cudaEventRecord(ev_packed, ss)) != cudaSuccess || (e = cudaStreamWaitEvent(sd, ev_packed, 0)) != cudaSuccess)
+    return cuda_fail(e, "order the re-send");
+  st = run_list(dst, kModeUnpack, dst->d_ids, n, buf, sd);
+  if (st != FR_OK) return st;
+  *failing = n;
+  return FR_OK;
 }
 
 }  // namespace
@@ -143,14 +402,16 @@ const char* fr_status_str(fr_status s) {
 
 const char* fr_last_error(void) { return g_err; }
 
-int fr_version(void) { return 10000; }
+int fr_version(void) { return 10100; }
 
-fr_status fr_plan_create(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes, fr_plan* out) {
+fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes,
+                                 uint32_t n_batches, fr_plan* out) {
   if (out == nullptr) return invalid("out is null");
   *out = nullptr;
   if (n_tensors > 0 && tensors == nullptr) return invalid("tensors is null");
   if (chunk_bytes == 0 || chunk_bytes % 4 != 0) return invalid("chunk_bytes must be a positive multiple of 4");
   if (n_tensors >= (1ull << 32)) return invalid("too many tensors");
+  if (n_batches == 0) return invalid("n_batches must be at least 1");
   uint64_t n_chunks = 0, state = 0;
   for (uint64_t t = 0; t < n_tensors; ++t) {
     const fr_tensor& x = tensors[t];
@@ -180,12 +441,12 @@ fr_status fr_plan_create(const fr_tensor* tensors, uint64_t n_tensors, uint64_t 
   p->chunk_bytes = chunk_bytes;
   p->n_chunks = n_chunks;
   p->state_bytes = state;
+  p->n_batches = static_cast<uint32_t>(std::max<uint64_t>(1, std::min<uint64_t>(n_batches, n_chunks)));
 
   // ---- chunks and packed layout
   p->chunks.resize(n_chunks);
   uint64_t payload = align_up(n_chunks * kHeaderBytes, kPayloadAlign);
   uint64_t c = 0;
-  uint64_t class_blocks[6] = {0, 0, 0, 0, 0, 0};
   for (uint64_t t = 0; t < n_tensors; ++t) {
     const bool aligned = (reinterpret_cast<uintptr_t>(tensors[t].ptr) % 16 == 0) && (chunk_bytes % 16 == 0);
     const uint32_t cls = tensors[t].dtype * 2 + (aligned ? 1 : 0);
@@ -196,75 +457,51 @@ fr_status fr_plan_create(const fr_tensor* tensors, uint64_t n_tensors, uint64_t 
       d.addr = reinterpret_cast<uint64_t>(tensors[t].ptr) + off;
       d.tensor_off = off;
       d.payload_off = payload;
-      d.blk_begin = class_blocks[cls];
       d.tensor_idx = static_cast<uint32_t>(t);
       d.dtype = tensors[t].dtype;
       d.sweep_class = cls;
+      d.seg_base = static_cast<uint32_t>(p->n_segs);
+      p->n_segs += (d.len / kBlockBytes + kSegBlocks - 1) / kSegBlocks;
       payload += align_up(d.len, kPayloadAlign);
-      class_blocks[cls] += d.len / kBlockBytes;
     }
   }
   p->packed_bytes = payload;
-
-  // ---- per class: equal block ranges per warp, one record per (warp, chunk)
-  // overlap.  Records are numbered class by class, so each chunk's records
-  // are consecutive.
-  std::vector<WarpDesc> warps;
-  std::vector<uint32_t> lists;
-  std::vector<uint64_t> rec_nblk;
-  const uint64_t W = static_cast<uint64_t>(n_sm) * kSweepWarps;
-  p->n_warps = static_cast<uint32_t>(W);
-  for (uint32_t cls = 0; cls < 6; ++cls) {
-    const uint64_t blk = class_blocks[cls];
-    if (blk == 0) continue;
-    SweepClass sc;
-    sc.dtype = cls / 2;
-    sc.aligned = (cls & 1u) != 0;
-    sc.n_blocks = blk;
-    sc.warp_off = warps.size();
-    sc.list_off = lists.size();
-    for (uint64_t i = 0; i < n_chunks; ++i)
-      if (p->chunks[i].sweep_class == cls && p->chunks[i].len >= static_cast<uint64_t>(kBlockBytes))
-        lists.push_back(static_cast<uint32_t>(i));
-    const uint32_t* list = lists.data() + sc.list_off;
-    uint64_t k = 0;  // walks the class list monotonically
-    for (uint64_t w = 0; w < W; ++w) {
-      const uint64_t b0 = blk * w / W, b1 = blk * (w + 1) / W;
-      WarpDesc wd;
-      std::memset(&wd, 0, sizeof wd);
-      wd.blk_begin = b0;
-      wd.nblk = b1 - b0;
-      wd.rec_base = static_cast<uint32_t>(rec_nblk.size());
-      if (b1 > b0) {
-        while (b0 >= p->chunks[list[k]].blk_begin + p->chunks[list[k]].len / kBlockBytes) ++k;
-        wd.first_chunk = static_cast<uint32_t>(k);
-        uint64_t b = b0, j = k;
-        while (b < b1) {
-          ChunkDesc& d = p->chunks[list[j]];
-          const uint64_t end = d.blk_begin + d.len / kBlockBytes;
-          const uint64_t n = std::min(b1, end) - b;
-          if (d.n_recs == 0) d.first_rec = static_cast<uint32_t>(rec_nblk.size());
-          d.n_recs += 1;
-          rec_nblk.push_back(n);
-          b += n;
-          if (b == end) ++j;
-        }
-      }
-      warps.push_back(wd);
-    }
-    p->classes.push_back(sc);
+  if (p->n_segs >= (1ull << 32)) {
+    delete p;
+    return invalid("state too large");
   }
-  p->n_recs = rec_nblk.size();
 
-  // ---- device tables
-  e = upload(&p->d_chunks, p->chunks);
-  if (e == cudaSuccess) e = upload(&p->d_warps, warps);
-  if (e == cudaSuccess) e = upload(&p->d_class_chunks, lists);
-  if (e == cudaSuccess) e = upload(&p->d_rec_nblk, rec_nblk);
-  if (e == cudaSuccess && p->n_recs) e = cudaMalloc(&p->d_recs, p->n_recs * sizeof(Record));
+  // ---- decompositions
+  e = cudaSuccess;
+  if (n_chunks > 0) {
+    e = build_decomp(p->chunks, {0, n_chunks}, n_sm, n_chunks, p->whole);
+    if (e == cudaSuccess && p->n_batches > 1) {
+      // batch starts at about equal state bytes, every batch non-empty
+      std::vector<uint64_t> bounds(1, 0);
+      uint64_t acc = 0, cc = 0;
+      for (uint32_t b = 1; b < p->n_batches; ++b) {
+        const uint64_t target = state / p->n_batches * b;
+        while (cc < n_chunks && (acc < target || cc <= bounds.back())) acc += p->chunks[cc++].len;
+        const uint64_t room = n_chunks - (p->n_batches - b);  // leave one chunk per later batch
+        bounds.push_back(std::min(cc, room));
+      }
+      bounds.push_back(n_chunks);
+      for (size_t i = 1; i < bounds.size(); ++i)
+        if (bounds[i] <= bounds[i - 1]) bounds[i] = bounds[i - 1] + 1;
+      e = build_decomp(p->chunks, bounds, std::max(1, n_sm / 2), 0, p->batched);
+    }
+  }
+  if (e == cudaSuccess && p->n_segs) e = cudaMalloc(&p->d_segs, p->n_segs * sizeof(double));
   if (e == cudaSuccess && n_chunks) e = cudaMalloc(&p->d_flags, n_chunks);
+  if (e == cudaSuccess && n_chunks) e = cudaMalloc(&p->d_ids, n_chunks * sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaMalloc(&p->d_count, sizeof(uint64_t));
   if (e == cudaSuccess) e = cudaMalloc(&p->d_status, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMemset(p->d_status, 0, sizeof(uint32_t));
+  for (uint32_t i = 0; e == cudaSuccess && i < p->n_batches + 1; ++i) {
+    cudaEvent_t ev;
+    e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+    if (e == cudaSuccess) p->events.push_back(ev);
+  }
   if (e != cudaSuccess) {
     free_device(p);
     delete p;
@@ -272,6 +509,10 @@ fr_status fr_plan_create(const fr_tensor* tensors, uint64_t n_tensors, uint64_t 
   }
   *out = p;
   return FR_OK;
+}
+
+fr_status fr_plan_create(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes, fr_plan* out) {
+  return fr_plan_create_batched(tensors, n_tensors, chunk_bytes, 1, out);
 }
 
 fr_status fr_plan_info(fr_plan p, uint64_t* n_chunks, uint64_t* packed_bytes, uint64_t* state_bytes) {
@@ -294,6 +535,21 @@ fr_status fr_plan_chunk(fr_plan p, uint64_t chunk_id, uint32_t* tensor_idx, uint
   return FR_OK;
 }
 
+fr_status fr_plan_batch(fr_plan p, uint32_t batch, uint32_t* n_batches, uint64_t* first_chunk, uint64_t* n_chunks) {
+  if (p == nullptr) return invalid("plan is null");
+  if (n_batches) *n_batches = p->n_chunks ? p->n_batches : 0;
+  if (p->n_chunks == 0) {
+    if (first_chunk) *first_chunk = 0;
+    if (n_chunks) *n_chunks = 0;
+    return FR_OK;
+  }
+  if (batch >= p->n_batches) return invalid("batch out of range");
+  const BatchInfo& b = batch_decomp(p).batches[batch];
+  if (first_chunk) *first_chunk = b.c_begin;
+  if (n_chunks) *n_chunks = b.c_end - b.c_begin;
+  return FR_OK;
+}
+
 void fr_plan_destroy(fr_plan p) {
   if (p == nullptr) return;
   DeviceGuard g(p->device);
@@ -302,63 +558,25 @@ void fr_plan_destroy(fr_plan p) {
   delete p;
 }
 
-static fr_status run_sweep(fr_plan p, int mode, uint8_t* packed, FpEntry* out_fp, cudaStream_t s) {
-  for (const SweepClass& sc : p->classes) {
-    SweepParams sp;
-    sp.chunks = p->d_chunks;
-    sp.warps = p->d_warps + sc.warp_off;
-    sp.class_chunks = p->d_class_chunks + sc.list_off;
-    sp.recs = p->d_recs;
-    sp.packed = packed;
-    sp.n_warps = p->n_warps;
-    cudaError_t e;
-    if (mode == kModeFingerprint)
-      e = launch_sweep_fp(sc.dtype, sc.aligned, sp, p->n_sm, s);
-    else if (mode == kModePack)
-      e = launch_sweep_pack(sc.dtype, sc.aligned, sp, p->n_sm, s);
-    else
-      e = launch_sweep_unpack(sc.dtype, sc.aligned, sp, p->n_sm, s);
-    if (e != cudaSuccess) return cuda_fail(e, "sweep kernel launch");
-  }
-  FinalizeParams fp;
-  fp.chunks = p->d_chunks;
-  fp.recs = p->d_recs;
-  fp.rec_nblk = p->d_rec_nblk;
-  fp.n_chunks = p->n_chunks;
-  fp.packed = packed;
-  fp.out_fp = out_fp;
-  fp.flags = p->d_flags;
-  cudaError_t e = launch_finalize(mode, fp, s);
-  if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
-  return FR_OK;
-}
-
 fr_status fr_fingerprint(fr_plan p, fr_fp* out_dev, void* stream) {
   if (p == nullptr) return invalid("plan is null");
   if (p->n_chunks == 0) return FR_OK;
   if (out_dev == nullptr) return invalid("out_dev is null");
   DeviceGuard g(p->device);
   if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
-  return run_sweep(p, kModeFingerprint, nullptr, reinterpret_cast<FpEntry*>(out_dev),
-                   static_cast<cudaStream_t>(stream));
+  return run_batches(p, p->whole, kModeFingerprint, nullptr, reinterpret_cast<FpEntry*>(out_dev), 0, 1,
+                     static_cast<cudaStream_t>(stream));
 }
 
 fr_status fr_pack(fr_plan p, void* dst, uint64_t dst_bytes, void* stream) {
   if (p == nullptr) return invalid("plan is null");
   if (p->n_chunks == 0) return FR_OK;
-  if (dst == nullptr) return invalid("dst is null");
-  if (reinterpret_cast<uintptr_t>(dst) % 16 != 0) {
-    set_err("packed buffer must be 16-byte aligned");
-    return FR_ERR_ALIGNMENT;
-  }
-  if (dst_bytes < p->packed_bytes) {
-    set_err("packed buffer holds %llu bytes, plan needs %llu", (unsigned long long)dst_bytes,
-            (unsigned long long)p->packed_bytes);
-    return FR_ERR_BUFFER_TOO_SMALL;
-  }
+  fr_status st = check_packed_buffer(p, dst, dst_bytes);
+  if (st != FR_OK) return st;
   DeviceGuard g(p->device);
   if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
-  return run_sweep(p, kModePack, static_cast<uint8_t*>(dst), nullptr, static_cast<cudaStream_t>(stream));
+  return run_batches(p, p->whole, kModePack, static_cast<uint8_t*>(dst), nullptr, 0, 1,
+                     static_cast<cudaStream_t>(stream));
 }
 
 fr_status fr_unpack_verify(fr_plan p, const void* src, uint64_t src_bytes, uint32_t* mismatch_dev, uint64_t cap,
@@ -373,20 +591,117 @@ fr_status fr_unpack_verify(fr_plan p, const void* src, uint64_t src_bytes, uint3
     cudaError_t e = cudaMemsetAsync(n_mismatch_dev, 0, sizeof(uint64_t), s);
     return e == cudaSuccess ? FR_OK : cuda_fail(e, "cudaMemsetAsync");
   }
-  if (src == nullptr) return invalid("src is null");
-  if (reinterpret_cast<uintptr_t>(src) % 16 != 0) {
-    set_err("packed buffer must be 16-byte aligned");
-    return FR_ERR_ALIGNMENT;
-  }
-  if (src_bytes < p->packed_bytes) {
-    set_err("packed buffer holds %llu bytes, plan needs %llu", (unsigned long long)src_bytes,
-            (unsigned long long)p->packed_bytes);
-    return FR_ERR_BUFFER_TOO_SMALL;
-  }
-  fr_status st = run_sweep(p, kModeUnpack, const_cast<uint8_t*>(static_cast<const uint8_t*>(src)), nullptr, s);
+  fr_status st = check_packed_buffer(p, src, src_bytes);
+  if (st != FR_OK) return st;
+  st = run_batches(p, p->whole, kModeUnpack, const_cast<uint8_t*>(static_cast<const uint8_t*>(src)), nullptr, 0, 1, s);
   if (st != FR_OK) return st;
   cudaError_t e = launch_compact_flags(p->d_flags, p->n_chunks, mismatch_dev, cap, n_mismatch_dev, p->d_status, s);
   return e == cudaSuccess ? FR_OK : cuda_fail(e, "compaction kernel launch");
+}
+
+fr_status fr_pack_batch(fr_plan p, uint32_t batch, void* dst, uint64_t dst_bytes, void* stream) {
+  if (p == nullptr) return invalid("plan is null");
+  if (p->n_chunks == 0) return FR_OK;
+  if (batch >= p->n_batches) return invalid("batch out of range");
+  fr_status st = check_packed_buffer(p, dst, dst_bytes);
+  if (st != FR_OK) return st;
+  DeviceGuard g(p->device);
+  if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
+  return run_batches(p, batch_decomp(p), kModePack, static_cast<uint8_t*>(dst), nullptr, batch, batch + 1,
+                     static_cast<cudaStream_t>(stream));
+}
+
+fr_status fr_unpack_verify_batch(fr_plan p, uint32_t batch, const void* src, uint64_t src_bytes, void* stream) {
+  if (p == nullptr) return invalid("plan is null");
+  if (p->n_chunks == 0) return FR_OK;
+  if (batch >= p->n_batches) return invalid("batch out of range");
+  fr_status st = check_packed_buffer(p, src, src_bytes);
+  if (st != FR_OK) return st;
+  DeviceGuard g(p->device);
+  if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
+  return run_batches(p, batch_decomp(p), kModeUnpack, const_cast<uint8_t*>(static_cast<const uint8_t*>(src)),
+                     nullptr, batch, batch + 1, static_cast<cudaStream_t>(stream));
+}
+
+fr_status fr_unpack_collect(fr_plan p, uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev,
+                            void* stream) {
+  if (p == nullptr) return invalid("plan is null");
+  if (n_mismatch_dev == nullptr) return invalid("n_mismatch_dev is null");
+  if (cap > 0 && mismatch_dev == nullptr) return invalid("mismatch_dev is null");
+  DeviceGuard g(p->device);
+  if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (p->n_chunks == 0)
+    e = cudaMemsetAsync(n_mismatch_dev, 0, sizeof(uint64_t), s);
+  else
+    e = launch_compact_flags(p->d_flags, p->n_chunks, mismatch_dev, cap, n_mismatch_dev, p->d_status, s);
+  return e == cudaSuccess ? FR_OK : cuda_fail(e, "compaction kernel launch");
+}
+
+fr_status fr_restore(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint32_t max_retries,
+                     uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev, void* stream_src,
+                     void* stream_dst) {
+  if (src == nullptr || dst == nullptr) return invalid("plan is null");
+  if (n_mismatch_dev == nullptr) return invalid("n_mismatch_dev is null");
+  if (cap > 0 && mismatch_dev == nullptr) return invalid("mismatch_dev is null");
+  fr_status st = check_same_layout(src, dst);
+  if (st != FR_OK) return st;
+  DeviceGuard g(dst->device);
+  if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
+  cudaStream_t ss = static_cast<cudaStream_t>(stream_src), sd = static_cast<cudaStream_t>(stream_dst);
+  if (src->n_chunks == 0) {
+    cudaError_t e = cudaMemsetAsync(n_mismatch_dev, 0, sizeof(uint64_t), sd);
+    return e == cudaSuccess ? FR_OK : cuda_fail(e, "cudaMemsetAsync");
+  }
+  st = check_packed_buffer(src, staging, staging_bytes);
+  if (st != FR_OK) return st;
+  uint8_t* buf = static_cast<uint8_t*>(staging);
+  const Decomp& DS = batch_decomp(src);
+  const Decomp& DD = batch_decomp(dst);
+  cudaError_t e;
+  // Pipeline: batch b is unpacked on the receiver's stream as soon as the
+  // replica's stream has packed it, while the replica packs batch b+1.
+  for (uint32_t b = 0; b < src->n_batches; ++b) {
+    st = run_batches(src, DS, kModePack, buf, nullptr, b, b + 1, ss);
+    if (st != FR_OK) return st;
+    if ((e = cudaEventRecord(src->events[b], ss)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    if ((e = cudaStreamWaitEvent(sd, src->events[b], 0)) != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+    st = run_batches(dst, DD, kModeUnpack, buf, nullptr, b, b + 1, sd);
+    if (st != FR_OK) return st;
+  }
+  // Retries: re-send only the chunks that failed, straight from the replica.
+  for (uint32_t r = 0; r < max_retries; ++r) {
+    uint64_t failing = 0;
+    st = resend_failed(src, dst, buf, ss, sd, &failing);
+    if (st != FR_OK) return st;
+    if (failing == 0) break;
+  }
+  // Everything queued on the replica's stream is ordered before what follows
+  // on the receiver's stream.
+  cudaEvent_t ev_end = src->events[src->n_batches];
+  if ((e = cudaEventRecord(ev_end, ss)) != cudaSuccess || (e = cudaStreamWaitEvent(sd, ev_end, 0)) != cudaSuccess)
+    return cuda_fail(e, "order the end of the restore");
+  e = launch_compact_flags(dst->d_flags, dst->n_chunks, mismatch_dev, cap, n_mismatch_dev, dst->d_status, sd);
+  return e == cudaSuccess ? FR_OK : cuda_fail(e, "compaction kernel launch");
+}
+
+fr_status fr_resend(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint64_t* n_resent,
+                    void* stream_src, void* stream_dst) {
+  if (src == nullptr || dst == nullptr) return invalid("plan is null");
+  fr_status st = check_same_layout(src, dst);
+  if (st != FR_OK) return st;
+  if (n_resent) *n_resent = 0;
+  if (src->n_chunks == 0) return FR_OK;
+  st = check_packed_buffer(src, staging, staging_bytes);
+  if (st != FR_OK) return st;
+  DeviceGuard g(dst->device);
+  if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
+  uint64_t n = 0;
+  st = resend_failed(src, dst, static_cast<uint8_t*>(staging), static_cast<cudaStream_t>(stream_src),
+                     static_cast<cudaStream_t>(stream_dst), &n);
+  if (n_resent) *n_resent = n;
+  return st;
 }
 
 fr_status fr_diff(const fr_fp* a_dev, const fr_fp* b_dev, uint64_t n_chunks, uint32_t* diverged_dev, uint64_t cap,

@@ -4,8 +4,9 @@
 // The sweep kernel leaves one record per piece (the part of a chunk body one
 // warp covered).  Here one warp per chunk:
 //   1. shifts each record's raw CRC to its position in the chunk and XORs them
-//      (raw(A||B) = raw(A) * x^(8|B|) ^ raw(B)), and sums the records' sums of
-//      squares and non-finite counts in record order;
+//      (raw(A||B) = raw(A) * x^(8|B|) ^ raw(B)), adds the records' non-finite
+//      counts, and adds the body's 16 KiB segment sums of squares in an order
+//      fixed by segment index (so the result does not depend on the plan);
 //   2. handles the chunk's tail (len % 512 bytes): lane l takes bytes
 //      [16l, 16l+16) of it, CRCs them a byte at a time, sums their squares in
 //      fp64, and copies them for pack/unpack;
@@ -90,27 +91,31 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
   __syncthreads();
   const uint32_t lane = threadIdx.x & 31u;
   const uint64_t stride = static_cast<uint64_t>(gridDim.x) * kFinWarps;
-  for (uint64_t c = static_cast<uint64_t>(blockIdx.x) * kFinWarps + (threadIdx.x >> 5); c < p.n_chunks;
-       c += stride) {
+  for (uint64_t pos = p.c_begin + static_cast<uint64_t>(blockIdx.x) * kFinWarps + (threadIdx.x >> 5);
+       pos < p.c_end; pos += stride) {
+    const uint64_t c = p.ids ? p.ids[pos] : pos;
     const ChunkDesc cd = p.chunks[c];
     const uint64_t body = cd.len & ~static_cast<uint64_t>(kBlockBytes - 1);
     const uint32_t tail = static_cast<uint32_t>(cd.len - body);
     const bool values = (MODE != kModeUnpack) && (cd.dtype != kDtBytes);
+    // list mode: one record per chunk with a body, at the list position
+    const uint64_t first_rec = p.ids ? pos : cd.first_rec;
+    const int64_t n_recs = p.ids ? (body ? 1 : 0) : cd.n_recs;
 
     // ---- 1. records, last batch first so the byte count after each is known
     uint32_t raw = 0;
     double sq_rec = 0.0;
     uint32_t nf_rec = 0;
     uint64_t carry = tail;
-    for (int64_t hi = cd.n_recs; hi > 0;) {
+    for (int64_t hi = n_recs; hi > 0;) {
       const int64_t lo = hi > 32 ? hi - 32 : 0;
       const int64_t i = lo + lane;
       const bool have = i < hi;
       Record rec{0u, 0u, 0.0};
       uint64_t len = 0;
       if (have) {
-        rec = p.recs[cd.first_rec + i];
-        len = p.rec_nblk[cd.first_rec + i] * kBlockBytes;
+        rec = p.recs[first_rec + i];
+        len = p.ids ? body : p.rec_nblk[first_rec + i] * kBlockBytes;
       }
       uint64_t suf = len;  // bytes of this record and the later ones in the batch
 #pragma unroll
@@ -120,16 +125,20 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
       }
       if (have) raw ^= shift_bytes(rec.crc, carry + suf - len);
       carry += __shfl_sync(kFull, suf, 0);
-      double s = rec.sumsq;
       uint32_t n = rec.nonfinite;
 #pragma unroll
-      for (int m = 16; m >= 1; m >>= 1) {
-        s += __shfl_down_sync(kFull, s, m);
-        n += __shfl_down_sync(kFull, n, m);
-      }
-      sq_rec += __shfl_sync(kFull, s, 0);
+      for (int m = 16; m >= 1; m >>= 1) n += __shfl_down_sync(kFull, n, m);
       nf_rec += __shfl_sync(kFull, n, 0);
       hi = lo;
+    }
+    // the body's segment sums, in an order fixed by segment index alone
+    if (values) {
+      const uint64_t n_seg = (body / kBlockBytes + kSegBlocks - 1) / kSegBlocks;
+      double s = 0.0;
+      for (uint64_t k = lane; k < n_seg; k += 32) s += p.segs[cd.seg_base + k];
+#pragma unroll
+      for (int m = 16; m >= 1; m >>= 1) s += __shfl_down_sync(kFull, s, m);
+      sq_rec = s;
     }
 
     // ---- 2. tail
@@ -334,8 +343,8 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(Pred pred, uin
 }  // namespace
 
 cudaError_t launch_finalize(int mode, const FinalizeParams& p, cudaStream_t s) {
-  if (p.n_chunks == 0) return cudaSuccess;
-  uint64_t want = (p.n_chunks + kFinWarps - 1) / kFinWarps;
+  if (p.c_end <= p.c_begin) return cudaSuccess;
+  uint64_t want = (p.c_end - p.c_begin + kFinWarps - 1) / kFinWarps;
   const int grid = static_cast<int>(want < 4096 ? want : 4096);
   if (mode == kModeFingerprint)
     finalize_kernel<kModeFingerprint><<<grid, kFinThreads, 0, s>>>(p);

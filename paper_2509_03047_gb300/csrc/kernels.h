@@ -16,6 +16,7 @@ struct SweepParams {
   const WarpDesc* warps;  // this class's per-warp ranges
   const uint32_t* class_chunks;  // ids of this class's chunks with a body, in order
   Record* recs;
+  double* segs;           // segment sums of squares (fingerprint, pack)
   uint8_t* packed;        // pack: destination; unpack: source; fingerprint: unused
   uint32_t n_warps;       // warps with a descriptor
 };
@@ -23,8 +24,11 @@ struct SweepParams {
 struct FinalizeParams {
   const ChunkDesc* chunks;
   const Record* recs;
+  const double* segs;
   const uint64_t* rec_nblk;
-  uint64_t n_chunks;
+  uint64_t n_chunks;        // chunks of the whole plan
+  uint64_t c_begin, c_end;  // chunks to finalize: [c_begin, c_end), or list positions if ids != null
+  const uint32_t* ids;      // list mode: chunk ids; the record of list position i is recs[i]
   uint8_t* packed;  // pack: destination; unpack: source
   FpEntry* out_fp;  // fingerprint: output table
   uint8_t* flags;   // unpack: per-chunk verdict
@@ -42,10 +46,26 @@ cudaError_t configure_sweep_fp();
 cudaError_t configure_sweep_pack();
 cudaError_t configure_sweep_unpack();
 
+// List mode: one warp per listed chunk sweeps its whole body into recs[i].
+struct ListParams {
+  const ChunkDesc* chunks;
+  const uint32_t* ids;
+  uint64_t n;
+  Record* recs;
+  double* segs;
+  uint8_t* packed;
+};
+
 // One class of chunks: element type and 16-byte alignment of its tensors.
 cudaError_t launch_sweep_fp(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
 cudaError_t launch_sweep_pack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
 cudaError_t launch_sweep_unpack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
+cudaError_t launch_list_pack(const ListParams& p, cudaStream_t s);
+cudaError_t launch_list_unpack(const ListParams& p, cudaStream_t s);
+inline cudaError_t launch_list_sweep(int mode, const ListParams& p, cudaStream_t s) {
+  return mode == kModePack ? launch_list_pack(p, s) : launch_list_unpack(p, s);
+}
+
 cudaError_t launch_finalize(int mode, const FinalizeParams& p, cudaStream_t s);
 // Ascending ids of the set flags, first `cap` of them, and the true count.
 cudaError_t launch_compact_flags(const uint8_t* flags, uint64_t n, uint32_t* out, uint64_t cap,

@@ -8,7 +8,7 @@
 // equal ranges, one per warp of that class's sweep kernel, so every warp moves
 // the same number of bytes whatever the tensor sizes.  A warp's range overlaps
 // one or more chunks; each overlap is a "piece" and produces one record (raw
-// CRC, non-finite count, sum of squares).
+// CRC, non-finite count).  Warp ranges start on segment boundaries.
 // The records of a chunk are consecutive and in order.  The finalize kernel
 // (one warp per chunk) folds a chunk's records and its tail.
 #pragma once
@@ -18,6 +18,16 @@
 namespace frk {
 
 constexpr uint64_t kHeaderBytes = 64;
+// A chunk body is cut into segments of kSegBlocks 512-byte blocks (16 KiB,
+// the last one shorter).  Each segment's sum of squares is computed in an
+// order fixed by positions alone and stored at its own index, and a chunk's
+// sum adds its segments in a fixed order: the result does not depend on how
+// the plan spreads the work over warps, batches or SMs.
+#ifndef FR_SEG_BLOCKS
+#define FR_SEG_BLOCKS 32
+#endif
+constexpr uint64_t kSegBlocks = FR_SEG_BLOCKS;
+static_assert((kSegBlocks & (kSegBlocks - 1)) == 0, "a power of two");
 constexpr uint64_t kPayloadAlign = 256;
 constexpr uint32_t kMagic = 0x31435246u;  // bytes 'F','R','C','1'
 constexpr uint32_t kVersion = 1;
@@ -35,7 +45,7 @@ struct ChunkDesc {       // 64 bytes
   uint32_t first_rec;    // records of this chunk: [first_rec, first_rec + n_recs)
   uint32_t n_recs;
   uint32_t sweep_class;  // dtype * 2 + (tensor 16-byte aligned ? 1 : 0)
-  uint32_t pad1;
+  uint32_t seg_base;     // index of the body's first segment sum
 };
 static_assert(sizeof(ChunkDesc) == 64, "ChunkDesc layout");
 
@@ -51,7 +61,7 @@ static_assert(sizeof(WarpDesc) == 32, "WarpDesc layout");
 struct Record {          // one piece's partial result
   uint32_t crc;          // raw CRC (preset 0, no final XOR) of the piece's bytes
   uint32_t nonfinite;
-  double sumsq;
+  double unused;         // sums of squares go to the segment array
 };
 static_assert(sizeof(Record) == 16, "Record layout");
 

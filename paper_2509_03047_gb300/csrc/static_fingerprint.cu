@@ -41,6 +41,7 @@ constexpr uint64_t kMaxWarpsPerClass = 160 * kSweepWarps;  // up to 160 SMs
 constexpr uint64_t kClasses = 6;
 constexpr uint64_t kMaxWarps = kClasses * kMaxWarpsPerClass;
 constexpr uint64_t kMaxRecs = kMaxWarps + kMaxChunks;
+constexpr uint64_t kMaxSegs = FR_STATIC_MAX_SEGMENTS;  // 16 KiB sum segments
 
 // Byte offsets of the tables inside the static array (256-byte aligned).
 constexpr uint64_t kOffChunks = 0;
@@ -48,7 +49,8 @@ constexpr uint64_t kOffLists = align_up(kOffChunks + kMaxChunks * sizeof(ChunkDe
 constexpr uint64_t kOffWarps = align_up(kOffLists + kMaxChunks * sizeof(uint32_t), 256);
 constexpr uint64_t kOffRecNblk = align_up(kOffWarps + kMaxWarps * sizeof(WarpDesc), 256);
 constexpr uint64_t kOffRecs = align_up(kOffRecNblk + kMaxRecs * sizeof(uint64_t), 256);
-constexpr uint64_t kScratchBytes = align_up(kOffRecs + kMaxRecs * sizeof(Record), 256);
+constexpr uint64_t kOffSegs = align_up(kOffRecs + kMaxRecs * sizeof(Record), 256);
+constexpr uint64_t kScratchBytes = align_up(kOffSegs + kMaxSegs * sizeof(double), 256);
 static_assert(kScratchBytes < (8ull << 20), "the static scratch must stay modest");
 
 // The device-side scratch.  In host code this name is only a stand-in for the
@@ -62,6 +64,7 @@ struct HostTables {
   uint32_t lists[kMaxChunks];
   WarpDesc warps[kMaxWarps];
   uint64_t rec_nblk[kMaxRecs];
+  uint64_t seg_start[kMaxSegs + 1];  // per class: block where each segment starts
 };
 HostTables g_host;
 std::mutex g_mu;
@@ -109,6 +112,13 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
     n_chunks += (x.nbytes + chunk_bytes - 1) / chunk_bytes;
     if (n_chunks > kMaxChunks) return fail(FR_ERR_INVALID_ARG, "more chunks than FR_STATIC_MAX_CHUNKS");
   }
+  uint64_t n_segs = 0;
+  for (uint64_t t = 0; t < n_tensors; ++t)
+    for (uint64_t off = 0; off < tensors[t].nbytes; off += chunk_bytes) {
+      const uint64_t len = std::min<uint64_t>(chunk_bytes, tensors[t].nbytes - off);
+      n_segs += (len / kBlockBytes + kSegBlocks - 1) / kSegBlocks;
+    }
+  if (n_segs > kMaxSegs) return fail(FR_ERR_INVALID_ARG, "more sum segments than FR_STATIC_MAX_SEGMENTS");
   if (n_chunks == 0) return FR_OK;
   if (out_dev == nullptr) return fail(FR_ERR_INVALID_ARG, "out_dev is null");
 
@@ -130,7 +140,7 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
   HostTables& h = g_host;
   uint64_t payload = align_up(n_chunks * kHeaderBytes, kPayloadAlign);
   uint64_t class_blocks[kClasses] = {0, 0, 0, 0, 0, 0};
-  uint64_t c = 0;
+  uint64_t c = 0, seg = 0;
   for (uint64_t t = 0; t < n_tensors; ++t) {
     const bool aligned = (reinterpret_cast<uintptr_t>(tensors[t].ptr) % 16 == 0) && (chunk_bytes % 16 == 0);
     const uint32_t cls = tensors[t].dtype * 2 + (aligned ? 1 : 0);
@@ -145,6 +155,8 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
       d.tensor_idx = static_cast<uint32_t>(t);
       d.dtype = tensors[t].dtype;
       d.sweep_class = cls;
+      d.seg_base = static_cast<uint32_t>(seg);
+      seg += (d.len / kBlockBytes + kSegBlocks - 1) / kSegBlocks;
       payload += align_up(d.len, kPayloadAlign);
       class_blocks[cls] += d.len / kBlockBytes;
     }
@@ -164,9 +176,17 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
       if (h.chunks[i].sweep_class == cls && h.chunks[i].len >= static_cast<uint64_t>(kBlockBytes))
         h.lists[n_lists++] = static_cast<uint32_t>(i);
     const uint32_t* list = h.lists + L.list_off;
+    // warp ranges start on 16 KiB segment boundaries (see layout.h)
+    uint64_t n_class_segs = 0;
+    for (uint64_t q = L.list_off; q < n_lists; ++q) {
+      const ChunkDesc& d = h.chunks[h.lists[q]];
+      const uint64_t nb = d.len / kBlockBytes;
+      for (uint64_t j = 0; j < nb; j += kSegBlocks) h.seg_start[n_class_segs++] = d.blk_begin + j;
+    }
+    h.seg_start[n_class_segs] = blk;
     uint64_t k = 0;
     for (uint64_t w = 0; w < W; ++w) {
-      const uint64_t b0 = blk * w / W, b1 = blk * (w + 1) / W;
+      const uint64_t b0 = h.seg_start[n_class_segs * w / W], b1 = h.seg_start[n_class_segs * (w + 1) / W];
       WarpDesc& wd = h.warps[n_warps++];
       std::memset(&wd, 0, sizeof wd);
       wd.blk_begin = b0;
@@ -209,6 +229,7 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
     sp.warps = reinterpret_cast<const WarpDesc*>(scratch + kOffWarps) + launches[i].warp_off;
     sp.class_chunks = reinterpret_cast<const uint32_t*>(scratch + kOffLists) + launches[i].list_off;
     sp.recs = d_recs;
+    sp.segs = reinterpret_cast<double*>(scratch + kOffSegs);
     sp.packed = nullptr;
     sp.n_warps = static_cast<uint32_t>(W);
     e = launch_sweep_fp(launches[i].dtype, launches[i].aligned, sp, n_sm, s);
@@ -217,8 +238,12 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
   FinalizeParams fp;
   fp.chunks = d_chunks;
   fp.recs = d_recs;
+  fp.segs = reinterpret_cast<const double*>(scratch + kOffSegs);
   fp.rec_nblk = reinterpret_cast<const uint64_t*>(scratch + kOffRecNblk);
   fp.n_chunks = n_chunks;
+  fp.c_begin = 0;
+  fp.c_end = n_chunks;
+  fp.ids = nullptr;
   fp.packed = nullptr;
   fp.out_fp = reinterpret_cast<FpEntry*>(out_dev);
   fp.flags = nullptr;

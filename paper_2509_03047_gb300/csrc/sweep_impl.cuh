@@ -47,7 +47,11 @@ namespace {
 constexpr int kWarps = kSweepWarps;
 constexpr int kThreads = kWarps * 32;
 constexpr int kTableBytes = 4 * 256 * 32 * 4;  // 4 tables x 256 entries x 32 lanes x 4 B
-// Pipeline geometry (compile-time; tuned on GB300 per mode).
+// Pipeline geometry (compile-time), tuned on GB300 by timing the 31.8 GB
+// Llama-70B shard.  The read-only fingerprint gains from bulk L2 prefetch one
+// span ahead; pack and unpack lose by it (their write stream evicts the
+// prefetched lines before use, and DRAM reads grow by ~20%), so they rely on
+// register stages alone, unpack with a deeper one.
 #ifndef FR_STAGE_FP
 #define FR_STAGE_FP 4
 #endif
@@ -55,23 +59,29 @@ constexpr int kTableBytes = 4 * 256 * 32 * 4;  // 4 tables x 256 entries x 32 la
 #define FR_STAGE_PACK 4
 #endif
 #ifndef FR_STAGE_UNPACK
-#define FR_STAGE_UNPACK 4
+#define FR_STAGE_UNPACK 8
 #endif
 #ifndef FR_AHEAD_FP
-#define FR_AHEAD_FP 2
+#define FR_AHEAD_FP 1
 #endif
 #ifndef FR_AHEAD_PACK
-#define FR_AHEAD_PACK 2
+#define FR_AHEAD_PACK 0
 #endif
 #ifndef FR_AHEAD_UNPACK
-#define FR_AHEAD_UNPACK 2
+#define FR_AHEAD_UNPACK 0
 #endif
-#ifndef FR_SWEEP_SPAN
-#define FR_SWEEP_SPAN 16
+#ifndef FR_LOADFIRST_FP
+#define FR_LOADFIRST_FP 0
 #endif
-// Blocks per validity span (a power of two, a multiple of every stage).
-constexpr int kSpan = FR_SWEEP_SPAN;
-static_assert((kSpan & (kSpan - 1)) == 0, "span geometry");
+#ifndef FR_LOADFIRST_PACK
+#define FR_LOADFIRST_PACK 0
+#endif
+#ifndef FR_LOADFIRST_UNPACK
+#define FR_LOADFIRST_UNPACK 1
+#endif
+// Blocks per validity span: one sum segment (a power of two, a multiple of
+// every stage).
+constexpr int kSpan = static_cast<int>(kSegBlocks);
 
 typedef unsigned long long u64;
 
@@ -292,11 +302,19 @@ __device__ __noinline__ bool span_is_zero(const uint8_t* sp, uint64_t b0, uint64
   return acc == 0;
 }
 
+// The span's sum as a double.  The four fp32 partial sums are first merged
+// error-free in fp32 (TwoSum), so only two conversions and one fp64 add reach
+// the narrow fp64 pipe; the error terms (about 2^-24 of the sum) are merged
+// with plain fp32 adds, which costs about 2^-48 relative.
 __device__ __forceinline__ double fold_to_double(const FpAcc& f) {
-  return ((static_cast<double>(lo_f(f.A)) + static_cast<double>(hi_f(f.A))) +
-          (static_cast<double>(lo_f(f.B)) + static_cast<double>(hi_f(f.B)))) +
-         ((static_cast<double>(lo_f(f.CA)) + static_cast<double>(hi_f(f.CA))) +
-          (static_cast<double>(lo_f(f.CB)) + static_cast<double>(hi_f(f.CB))));
+  u64 s = f.A, c = add2(f.CA, f.CB);
+  two_sum_acc(s, c, f.B);  // s + c == A + B + CA + CB up to the rounding of c
+  const float a = lo_f(s), b = hi_f(s);
+  const float t = a + b;  // scalar TwoSum of the two halves
+  const float z = t - a;
+  const float err = (a - (t - z)) + (b - z);
+  const float lo = (lo_f(c) + hi_f(c)) + err;
+  return static_cast<double>(t) + static_cast<double>(lo);
 }
 
 // ------------------------------------------------------------------ piece
@@ -314,18 +332,19 @@ struct Geo {
                                                                                               : FR_STAGE_UNPACK);
   static constexpr int kAhead = MODE == kModeFingerprint ? FR_AHEAD_FP : (MODE == kModePack ? FR_AHEAD_PACK
                                                                                               : FR_AHEAD_UNPACK);
+  // Issue a unit's reload before consuming it (more load lead, one register
+  // copy) or after (no copy): latency-bound modes want the former.
+  static constexpr bool kLoadFirst = MODE == kModeFingerprint ? FR_LOADFIRST_FP
+                                     : (MODE == kModePack ? FR_LOADFIRST_PACK : FR_LOADFIRST_UNPACK);
   static_assert(kSpan % kStage == 0, "a span holds whole stages");
 };
 
 // State of one lane while it sweeps a piece.
 template <int MODE, int DT>
 struct Lane {
-  uint32_t s[4];   // CRC streams 4l..4l+3
-  FpAcc f, snap;   // running fp32 sums and their value at the span start
-  double d;        // flushed sums
+  uint32_t s[4];  // CRC streams 4l..4l+3
+  FpAcc f;        // fp32 sums of the current span
   uint32_t nonfinite;
-  bool big;        // d already holds a sum >= 2^-60
-  int fold;
 };
 
 template <int MODE, int DT, int DAL>
@@ -339,28 +358,30 @@ __device__ __forceinline__ void do_unit(Lane<MODE, DT>& L, const uint4& v, uint8
   if (kFp) fp_unit<DT>(v, L.f);
 }
 
-// End of a span [b0, b1): the fast sums are kept if finite and either large
-// enough that fp32 underflow is negligible (below 2^-80 relative) or made of
-// zeros only; otherwise the span is redone exactly from a reload.
+// End of a span [b0, b1) (one segment): the fast sums are kept if finite and
+// either large enough that fp32 underflow is negligible (below 2^-77 relative)
+// or made of zeros only; otherwise the segment is summed exactly from a
+// reload.  The lanes' sums are then added in a fixed tree and lane 0 stores
+// the segment's sum at its index.
 template <int MODE, int DT, int SAL>
-__device__ __forceinline__ void span_end(Lane<MODE, DT>& L, const uint8_t* sp, uint64_t b0, uint64_t b1) {
-  constexpr int kFoldSpans = (DT == kDtF32 ? 128 : 64) / kSpan;  // <= 128 terms per f32x2 lane
+__device__ __forceinline__ void span_end(Lane<MODE, DT>& L, const uint8_t* sp, uint64_t b0, uint64_t b1,
+                                         double* seg, uint32_t lane) {
   const u64 ab = add2(L.f.A, L.f.B);
   const float tot = lo_f(ab) + hi_f(ab);
   bool ok = tot < __int_as_float(0x7F800000);
-  if (ok && !(tot >= 0x1p-60f) && !L.big) ok = span_is_zero<DT, SAL>(sp, b0, b1);
-  if (!ok) {
-    L.f = L.snap;
+  if (ok && !(tot >= 0x1p-60f)) ok = span_is_zero<DT, SAL>(sp, b0, b1);
+  double d;
+  if (ok) {
+    d = fold_to_double(L.f);
+  } else {
     const Exact x = slow_span<DT, SAL>(sp, b0, b1);
-    L.d += x.d;
+    d = x.d;
     L.nonfinite += x.nonfinite;
   }
-  if (++L.fold == kFoldSpans) {
-    L.d += fold_to_double(L.f);
-    L.big = L.big || (L.d >= 0x1p-60);
-    L.f.A = L.f.CA = L.f.B = L.f.CB = 0ull;
-    L.fold = 0;
-  }
+  L.f.A = L.f.CA = L.f.B = L.f.CB = 0ull;
+#pragma unroll
+  for (int m = 16; m >= 1; m >>= 1) d += __shfl_down_sync(0xFFFFFFFFu, d, m);
+  if (lane == 0) *seg = d;
 }
 
 // One piece: `nblk` 512-byte blocks from `src` (to `dst` for pack/unpack).
@@ -368,12 +389,12 @@ __device__ __forceinline__ void span_end(Lane<MODE, DT>& L, const uint8_t* sp, u
 //
 // Pipeline: lane 0 prefetches whole spans into L2 kAhead spans ahead with the
 // bulk-copy unit; each lane keeps kStage 16-byte units of the next stage in
-// flight in registers, which therefore mostly wait for L2.  The sums' validity
-// is checked once per span; a failing span is rolled back to its snapshot and
-// redone exactly from a reload.
+// flight in registers, which therefore mostly wait for L2.  Each span is one
+// sum segment: its fp32 sums start at zero, are checked at its end, and are
+// replaced by an exact sum from a reload when they fail.
 template <int MODE, int DT, int SAL, int DAL>
 __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
-                                            uint64_t nblk, uint32_t lane, Record* rec) {
+                                            uint64_t nblk, uint32_t lane, Record* rec, double* segs) {
   constexpr bool kFp = (MODE != kModeUnpack) && (DT != kDtBytes);
   constexpr int kStage = Geo<MODE>::kStage;
   constexpr int kAhead = Geo<MODE>::kAhead;
@@ -390,11 +411,7 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
   Lane<MODE, DT> L;
   L.s[0] = L.s[1] = L.s[2] = L.s[3] = 0;
   L.f = FpAcc{0ull, 0ull, 0ull, 0ull};
-  L.snap = L.f;
-  L.d = 0.0;
   L.nonfinite = 0;
-  L.big = false;
-  L.fold = 0;
 
   uint4 cur[kStage];
 #pragma unroll
@@ -403,44 +420,49 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
   const uint8_t* lp = sp + kStageBytes;  // the next stage's loads
 
   uint64_t i = 0;
-  // Steady state: this stage and the next are whole, so no predicates.
-  for (; i + 2 * kStage <= nblk; i += kStage) {
-    if ((i & (kSpan - 1)) == 0) {
-      if (kFp) L.snap = L.f;
-      if (kAhead > 0 && SAL == 16 && lane == 0) {
-        const uint64_t pf = i + kSpan * kAhead;
-        if (pf < nblk) {
-          const uint64_t n = (nblk - pf < kSpan) ? nblk - pf : kSpan;
-          prefetch_l2(src + pf * kBlockBytes, static_cast<uint32_t>(n * kBlockBytes));
-        }
+  // Steady state: whole spans whose following stage is whole too.  The inner
+  // stage loop has no branch at all; the span's prefetch and validity check
+  // sit outside it.
+  for (; i + kSpan + kStage <= nblk; i += kSpan) {
+    if (kAhead > 0 && SAL == 16 && lane == 0) {
+      const uint64_t pf = i + kSpan * kAhead;
+      if (pf < nblk) {
+        const uint64_t n = (nblk - pf < kSpan) ? nblk - pf : kSpan;
+        prefetch_l2(src + pf * kBlockBytes, static_cast<uint32_t>(n * kBlockBytes));
       }
     }
+#pragma unroll 1
+    for (int st = 0; st < kSpan / kStage; ++st) {
 #pragma unroll
-    for (int u = 0; u < kStage; ++u) {
-      const uint4 v = cur[u];
-      cur[u] = ld_unit<SAL>(lp + u * kBlockBytes);
-      do_unit<MODE, DT, DAL>(L, v, wp + u * kBlockBytes, lb);
+      for (int u = 0; u < kStage; ++u) {
+        if (Geo<MODE>::kLoadFirst) {
+          const uint4 v = cur[u];
+          cur[u] = ld_unit<SAL>(lp + u * kBlockBytes);
+          do_unit<MODE, DT, DAL>(L, v, wp + u * kBlockBytes, lb);
+        } else {
+          do_unit<MODE, DT, DAL>(L, cur[u], wp + u * kBlockBytes, lb);
+          cur[u] = ld_unit<SAL>(lp + u * kBlockBytes);
+        }
+      }
+      lp += kStageBytes;
+      wp += kStageBytes;
     }
-    lp += kStageBytes;
-    wp += kStageBytes;
-    if (kFp && ((i + kStage) & (kSpan - 1)) == 0) span_end<MODE, DT, SAL>(L, sp, i + kStage - kSpan, i + kStage);
+    if (kFp) span_end<MODE, DT, SAL>(L, sp, i, i + kSpan, segs + i / kSpan, lane);
   }
-  // Drain: the last one or two stages, the last possibly partial.
+  // Drain: the last (partial) span and the stage after it, with predicates.
   for (; i < nblk; i += kStage) {
-    if ((i & (kSpan - 1)) == 0 && kFp) L.snap = L.f;
 #pragma unroll
     for (int u = 0; u < kStage; ++u) {
       if (i + u < nblk) {
-        const uint4 v = cur[u];
+        do_unit<MODE, DT, DAL>(L, cur[u], wp + u * kBlockBytes, lb);
         if (i + kStage + u < nblk) cur[u] = ld_unit<SAL>(lp + u * kBlockBytes);
-        do_unit<MODE, DT, DAL>(L, v, wp + u * kBlockBytes, lb);
       }
     }
     lp += kStageBytes;
     wp += kStageBytes;
     const uint64_t end = (i + kStage < nblk) ? i + kStage : nblk;
     if (kFp && ((end & (kSpan - 1)) == 0 || end == nblk))
-      span_end<MODE, DT, SAL>(L, sp, i & ~static_cast<uint64_t>(kSpan - 1), end);
+      span_end<MODE, DT, SAL>(L, sp, i & ~static_cast<uint64_t>(kSpan - 1), end, segs + i / kSpan, lane);
   }
 
   // ---- fold the 128 streams into the raw CRC of the piece
@@ -461,32 +483,27 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
     v = mulk<gf_xpow(2048)>(v) ^ o;
   }
 
-  double d = L.d;
   uint32_t nonfinite = L.nonfinite;
   if (kFp) {
-    d += fold_to_double(L.f);
 #pragma unroll
-    for (int m = 16; m >= 1; m >>= 1) {
-      d += __shfl_down_sync(0xFFFFFFFFu, d, m);
-      nonfinite += __shfl_down_sync(0xFFFFFFFFu, nonfinite, m);
-    }
+    for (int m = 16; m >= 1; m >>= 1) nonfinite += __shfl_down_sync(0xFFFFFFFFu, nonfinite, m);
   }
   if (lane == 0) {
     Record r;
     r.crc = mulk<kUnbraid>(v);
     r.nonfinite = nonfinite;
-    r.sumsq = d;
+    r.unused = 0.0;
     *rec = r;
   }
 }
 
 template <int MODE, int DT, int AL>
 __device__ __forceinline__ void sweep_piece_al(const uint8_t* tensor, uint8_t* packed, uint64_t n,
-                                               uint32_t lane, Record* rec) {
+                                               uint32_t lane, Record* rec, double* segs) {
   if (MODE == kModeUnpack)
-    sweep_piece<MODE, DT, 16, AL>(packed, const_cast<uint8_t*>(tensor), n, lane, rec);
+    sweep_piece<MODE, DT, 16, AL>(packed, const_cast<uint8_t*>(tensor), n, lane, rec, segs);
   else
-    sweep_piece<MODE, DT, AL, 16>(tensor, packed, n, lane, rec);
+    sweep_piece<MODE, DT, AL, 16>(tensor, packed, n, lane, rec, segs);
 }
 
 // One kernel per (mode, element type, alignment class).  ALIGNED: every
@@ -509,18 +526,69 @@ __global__ void __launch_bounds__(kThreads, 1) sweep_kernel(SweepParams p) {
     const uint64_t n = (left < nb - off) ? left : nb - off;
     const uint8_t* tensor = reinterpret_cast<const uint8_t*>(cd.addr) + off * kBlockBytes;
     uint8_t* packed = (MODE == kModeFingerprint) ? nullptr : p.packed + cd.payload_off + off * kBlockBytes;
+    double* segs = p.segs + cd.seg_base + off / kSegBlocks;
     if (ALIGNED) {
-      sweep_piece_al<MODE, DT, 16>(tensor, packed, n, lane, p.recs + r);
+      sweep_piece_al<MODE, DT, 16>(tensor, packed, n, lane, p.recs + r, segs);
     } else if ((reinterpret_cast<uintptr_t>(tensor) & 3u) == 0) {
-      sweep_piece_al<MODE, DT, 4>(tensor, packed, n, lane, p.recs + r);
+      sweep_piece_al<MODE, DT, 4>(tensor, packed, n, lane, p.recs + r, segs);
     } else {
-      sweep_piece_al<MODE, DT, 1>(tensor, packed, n, lane, p.recs + r);
+      sweep_piece_al<MODE, DT, 1>(tensor, packed, n, lane, p.recs + r, segs);
     }
     ++r;
     b += n;
     left -= n;
     ++k;
   }
+}
+
+// List mode (re-sending failed chunks): warp w sweeps the whole body of chunk
+// ids[w] into recs[w].  Every variant is a separate function, so this cold
+// kernel's dispatch does not burden the registers of the hot ones.
+template <int MODE, int DT, bool ALIGNED>
+__device__ __noinline__ void list_piece(const uint8_t* tensor, uint8_t* packed, uint64_t n, uint32_t lane,
+                                        Record* rec, double* segs) {
+  if (ALIGNED)
+    sweep_piece_al<MODE, DT, 16>(tensor, packed, n, lane, rec, segs);
+  else if ((reinterpret_cast<uintptr_t>(tensor) & 3u) == 0)
+    sweep_piece_al<MODE, DT, 4>(tensor, packed, n, lane, rec, segs);
+  else
+    sweep_piece_al<MODE, DT, 1>(tensor, packed, n, lane, rec, segs);
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 1) list_kernel(ListParams p) {
+  fill_tables();
+  __syncthreads();
+  const uint32_t lane = threadIdx.x & 31u;
+  const uint64_t w = static_cast<uint64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+  if (w >= p.n) return;
+  const ChunkDesc cd = p.chunks[p.ids[w]];
+  const uint64_t nb = cd.len / kBlockBytes;
+  if (nb == 0) return;
+  const uint8_t* tensor = reinterpret_cast<const uint8_t*>(cd.addr);
+  uint8_t* packed = (MODE == kModeFingerprint) ? nullptr : p.packed + cd.payload_off;
+  const bool aligned = (cd.sweep_class & 1u) != 0;
+  const uint32_t dt = (MODE == kModeUnpack) ? kDtBytes : cd.dtype;
+  double* segs = p.segs + cd.seg_base;
+  Record* rec = p.recs + w;
+  if (dt == kDtF32) {
+    if (aligned) list_piece<MODE, kDtF32, true>(tensor, packed, nb, lane, rec, segs);
+    else list_piece<MODE, kDtF32, false>(tensor, packed, nb, lane, rec, segs);
+  } else if (dt == kDtBf16) {
+    if (aligned) list_piece<MODE, kDtBf16, true>(tensor, packed, nb, lane, rec, segs);
+    else list_piece<MODE, kDtBf16, false>(tensor, packed, nb, lane, rec, segs);
+  } else {
+    if (aligned) list_piece<MODE, kDtBytes, true>(tensor, packed, nb, lane, rec, segs);
+    else list_piece<MODE, kDtBytes, false>(tensor, packed, nb, lane, rec, segs);
+  }
+}
+
+template <int MODE>
+cudaError_t launch_list(const ListParams& p, cudaStream_t s) {
+  if (p.n == 0) return cudaSuccess;
+  const uint64_t ctas = (p.n + kWarps - 1) / kWarps;
+  list_kernel<MODE><<<static_cast<unsigned>(ctas), kThreads, kTableBytes, s>>>(p);
+  return cudaGetLastError();
 }
 
 template <int MODE, int DT, bool ALIGNED>
@@ -541,7 +609,8 @@ cudaError_t launch_one(const SweepParams& p, int n_ctas, cudaStream_t s) {
 // element type: it only checksums and copies).
 template <int MODE>
 cudaError_t configure_mode() {
-  cudaError_t e = configure_one<MODE, kDtBytes, true>();
+  cudaError_t e = cudaFuncSetAttribute(list_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTableBytes);
+  if (e == cudaSuccess) e = configure_one<MODE, kDtBytes, true>();
   if (e == cudaSuccess) e = configure_one<MODE, kDtBytes, false>();
   if (MODE != kModeUnpack) {
     if (e == cudaSuccess) e = configure_one<MODE, kDtBf16, true>();

@@ -9,4 +9,6 @@ cudaError_t launch_sweep_pack(uint32_t dtype, bool aligned, const SweepParams& p
   return launch_mode<kModePack>(dtype, aligned, p, n_ctas, s);
 }
 
+cudaError_t launch_list_pack(const ListParams& p, cudaStream_t s) { return launch_list<kModePack>(p, s); }
+
 }  // namespace frk

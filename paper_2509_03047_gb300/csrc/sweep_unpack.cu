@@ -9,4 +9,6 @@ cudaError_t launch_sweep_unpack(uint32_t dtype, bool aligned, const SweepParams&
   return launch_mode<kModeUnpack>(dtype, aligned, p, n_ctas, s);
 }
 
+cudaError_t launch_list_unpack(const ListParams& p, cudaStream_t s) { return launch_list<kModeUnpack>(p, s); }
+
 }  // namespace frk

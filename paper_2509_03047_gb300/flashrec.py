@@ -60,13 +60,22 @@ def _load() -> ctypes.CDLL:
     L.fr_diff.argtypes = [vp, vp, u64, vp, u64, vp, vp]
     L.fr_sync_status.argtypes = [vp, vp]
     L.fr_fingerprint_static.argtypes = [ctypes.POINTER(fr_tensor), u64, u64, vp, vp]
+    L.fr_plan_create_batched.argtypes = [ctypes.POINTER(fr_tensor), u64, u64, u32, ctypes.POINTER(vp)]
+    L.fr_plan_batch.argtypes = [vp, u32, ctypes.POINTER(u32), u64p, u64p]
+    L.fr_pack_batch.argtypes = [vp, u32, vp, u64, vp]
+    L.fr_unpack_verify_batch.argtypes = [vp, u32, vp, u64, vp]
+    L.fr_unpack_collect.argtypes = [vp, vp, u64, vp, vp]
+    L.fr_resend.argtypes = [vp, vp, vp, u64, u64p, vp, vp]
+    L.fr_restore.argtypes = [vp, vp, vp, u64, u32, vp, u64, vp, vp, vp]
     L.fr_status_str.argtypes = [ctypes.c_int]
     L.fr_status_str.restype = ctypes.c_char_p
     L.fr_last_error.argtypes = []
     L.fr_last_error.restype = ctypes.c_char_p
     L.fr_version.argtypes = []
     for name in ["fr_plan_create", "fr_plan_info", "fr_plan_chunk", "fr_fingerprint", "fr_pack",
-                 "fr_unpack_verify", "fr_diff", "fr_sync_status", "fr_version", "fr_fingerprint_static"]:
+                 "fr_unpack_verify", "fr_diff", "fr_sync_status", "fr_version", "fr_fingerprint_static",
+                 "fr_plan_create_batched", "fr_plan_batch", "fr_pack_batch", "fr_unpack_verify_batch",
+                 "fr_unpack_collect", "fr_resend", "fr_restore"]:
         getattr(L, name).restype = ctypes.c_int
     return L
 
@@ -108,8 +117,7 @@ def fr_dtype_of(t: torch.Tensor) -> int:
 
 # ---------------------------------------------------------------- C names
 
-def fr_plan_create(tensors: Sequence[torch.Tensor], chunk_bytes: int, dtypes: Optional[Sequence[int]] = None):
-    """Plan over contiguous CUDA tensors.  Returns the opaque handle (int)."""
+def _tensor_array(tensors, dtypes=None):
     arr = (fr_tensor * max(1, len(tensors)))()
     for i, t in enumerate(tensors):
         if t.numel() and not t.is_cuda:
@@ -120,9 +128,60 @@ def fr_plan_create(tensors: Sequence[torch.Tensor], chunk_bytes: int, dtypes: Op
         arr[i].nbytes = t.numel() * t.element_size()
         arr[i].dtype = dtypes[i] if dtypes is not None else fr_dtype_of(t)
         arr[i].flags = 0
+    return arr
+
+
+def fr_plan_create(tensors: Sequence[torch.Tensor], chunk_bytes: int, dtypes: Optional[Sequence[int]] = None):
+    """Plan over contiguous CUDA tensors.  Returns the opaque handle (int)."""
     h = ctypes.c_void_p()
-    _check(lib.fr_plan_create(arr, len(tensors), chunk_bytes, ctypes.byref(h)), "fr_plan_create")
+    _check(lib.fr_plan_create(_tensor_array(tensors, dtypes), len(tensors), chunk_bytes, ctypes.byref(h)),
+           "fr_plan_create")
     return h.value
+
+
+def fr_plan_create_batched(tensors: Sequence[torch.Tensor], chunk_bytes: int, n_batches: int,
+                           dtypes: Optional[Sequence[int]] = None):
+    h = ctypes.c_void_p()
+    _check(lib.fr_plan_create_batched(_tensor_array(tensors, dtypes), len(tensors), chunk_bytes, n_batches,
+                                      ctypes.byref(h)), "fr_plan_create_batched")
+    return h.value
+
+
+def fr_plan_batch(plan, batch: int):
+    nb, first, n = ctypes.c_uint32(), ctypes.c_uint64(), ctypes.c_uint64()
+    _check(lib.fr_plan_batch(plan, batch, ctypes.byref(nb), ctypes.byref(first), ctypes.byref(n)), "fr_plan_batch")
+    return nb.value, first.value, n.value
+
+
+def fr_pack_batch(plan, batch: int, dst: torch.Tensor, stream=None) -> None:
+    _check(lib.fr_pack_batch(plan, batch, dst.data_ptr() if dst.numel() else None, dst.numel(), _stream(stream)),
+           "fr_pack_batch")
+
+
+def fr_unpack_verify_batch(plan, batch: int, src: torch.Tensor, stream=None) -> None:
+    _check(lib.fr_unpack_verify_batch(plan, batch, src.data_ptr() if src.numel() else None, src.numel(),
+                                      _stream(stream)), "fr_unpack_verify_batch")
+
+
+def fr_unpack_collect(plan, mismatch: Optional[torch.Tensor], count: torch.Tensor, stream=None) -> None:
+    cap = 0 if mismatch is None else mismatch.numel()
+    _check(lib.fr_unpack_collect(plan, mismatch.data_ptr() if cap else None, cap, count.data_ptr(), _stream(stream)),
+           "fr_unpack_collect")
+
+
+def fr_resend(src_plan, dst_plan, staging: torch.Tensor, stream_src=None, stream_dst=None) -> int:
+    n = ctypes.c_uint64()
+    _check(lib.fr_resend(src_plan, dst_plan, staging.data_ptr() if staging.numel() else None, staging.numel(),
+                         ctypes.byref(n), _stream(stream_src), _stream(stream_dst)), "fr_resend")
+    return n.value
+
+
+def fr_restore(src_plan, dst_plan, staging: torch.Tensor, max_retries: int, mismatch: Optional[torch.Tensor],
+               count: torch.Tensor, stream_src=None, stream_dst=None) -> None:
+    cap = 0 if mismatch is None else mismatch.numel()
+    _check(lib.fr_restore(src_plan, dst_plan, staging.data_ptr() if staging.numel() else None, staging.numel(),
+                          max_retries, mismatch.data_ptr() if cap else None, cap, count.data_ptr(),
+                          _stream(stream_src), _stream(stream_dst)), "fr_restore")
 
 
 def fr_plan_info(plan):
@@ -211,11 +270,15 @@ def fp_view(table: torch.Tensor):
 class Plan:
     """A plan over a list of CUDA tensors, with allocation helpers."""
 
-    def __init__(self, tensors: Sequence[torch.Tensor], chunk_bytes: int):
+    def __init__(self, tensors: Sequence[torch.Tensor], chunk_bytes: int, n_batches: int = 1):
         self.tensors: List[torch.Tensor] = list(tensors)
         self.chunk_bytes = chunk_bytes
         self.device = self.tensors[0].device if self.tensors else torch.device("cuda", torch.cuda.current_device())
-        self.handle = fr_plan_create(self.tensors, chunk_bytes)
+        if n_batches > 1:
+            self.handle = fr_plan_create_batched(self.tensors, chunk_bytes, n_batches)
+        else:
+            self.handle = fr_plan_create(self.tensors, chunk_bytes)
+        self.n_batches = fr_plan_batch(self.handle, 0)[0] if n_batches > 1 else 1
         self.n_chunks, self.packed_bytes, self.state_bytes = fr_plan_info(self.handle)
 
     def close(self) -> None:
