@@ -200,6 +200,45 @@ fr_status fr_restore(fr_plan src, fr_plan dst, void* staging, uint64_t staging_b
                      uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev, void* stream_src,
                      void* stream_dst);
 
+/* ---------------------------------------------------------------- sharded (ZeRO / FSDP) state */
+
+/* With ZeRO / FSDP every data-parallel rank keeps only a shard of the
+ * flattened model states (Sec. III-A; ZeRO/FSDP panel of the restoration
+ * figure in Sec. III-E).  When the surviving copies are sharded another way
+ * (another data-parallel degree, another ZeRO group), no single peer holds a
+ * restarted rank's shard: it is assembled from pieces of several peers'
+ * shards.
+ *
+ * Sharding rule: a flat group of `n_elems` elements of `elem_bytes` bytes
+ * split `n` ways gives shard r the elements [r*q, min((r+1)*q, n_elems)),
+ * q = ceil(n_elems / n); shards past the end are empty.  (ZeRO/FSDP pad the
+ * group to a multiple of n; padding bytes are not model state and are not
+ * moved.)
+ *
+ * fr_shard_pieces lists, in ascending order, where shard `rank` of the group
+ * split `n_dst` ways lies among the shards of the same group split `n_src`
+ * ways: for each piece the source shard, the byte offset in that source
+ * shard, the byte offset in the destination shard and the byte count.  A
+ * non-empty shard has between 1 and n_src pieces.  *n_pieces always receives
+ * the true count; at most `cap` pieces are written, FR_ERR_CAPACITY if there
+ * are more.  Host only: no device work.
+ *
+ * A plan over the pieces' source regions (tensors inside several peers'
+ * shards) and a plan over their destination regions have the same layout, so
+ * one fr_restore between them assembles the whole shard from all its
+ * sources, and fr_fingerprint of both plans followed by fr_diff confirms that
+ * the result matches every source.
+ * Errors: FR_ERR_INVALID_ARG, FR_ERR_CAPACITY. */
+typedef struct {
+  uint32_t source;  /* source shard index, < n_src                */
+  uint32_t reserved;
+  uint64_t src_off; /* byte offset in the source shard             */
+  uint64_t dst_off; /* byte offset in the destination shard        */
+  uint64_t nbytes;  /* bytes in the piece (a multiple of elem_bytes) */
+} fr_piece;
+fr_status fr_shard_pieces(uint64_t n_elems, uint32_t elem_bytes, uint32_t n_dst, uint32_t rank, uint32_t n_src,
+                          fr_piece* out, uint64_t cap, uint64_t* n_pieces);
+
 /* ---------------------------------------------------------------- no allocation */
 
 /* The paper has no counterpart to this call; it serves callers that cannot

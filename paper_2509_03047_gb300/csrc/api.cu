@@ -738,4 +738,39 @@ fr_status fr_sync_status(fr_plan p, void* stream) {
   return FR_ERR_CAPACITY;
 }
 
+fr_status fr_shard_pieces(uint64_t n_elems, uint32_t elem_bytes, uint32_t n_dst, uint32_t rank, uint32_t n_src,
+                          fr_piece* out, uint64_t cap, uint64_t* n_pieces) {
+  if (n_pieces == nullptr) return invalid("n_pieces is null");
+  if (elem_bytes == 0 || n_dst == 0 || n_src == 0) return invalid("elem_bytes, n_dst and n_src must be positive");
+  if (rank >= n_dst) return invalid("rank must be below n_dst");
+  if (cap > 0 && out == nullptr) return invalid("out is null");
+  if (n_elems > UINT64_MAX / elem_bytes) return invalid("the flat group exceeds 2^64 bytes");
+  // Every shard holds ceil(n / shards) elements, the last non-empty one the rest.
+  const uint64_t per_dst = n_elems / n_dst + (n_elems % n_dst != 0);
+  const uint64_t per_src = n_elems / n_src + (n_elems % n_src != 0);
+  const uint64_t a = std::min<uint64_t>(static_cast<uint64_t>(rank) * per_dst, n_elems);
+  const uint64_t b = std::min<uint64_t>(a + per_dst, n_elems);
+  uint64_t n = 0;
+  if (a < b) {
+    for (uint64_t j = a / per_src; j * per_src < b; ++j) {
+      const uint64_t lo = std::max(a, j * per_src), hi = std::min(b, (j + 1) * per_src);
+      if (n < cap) {
+        fr_piece& pc = out[n];
+        pc.source = static_cast<uint32_t>(j);
+        pc.reserved = 0;
+        pc.src_off = (lo - j * per_src) * elem_bytes;
+        pc.dst_off = (lo - a) * elem_bytes;
+        pc.nbytes = (hi - lo) * elem_bytes;
+      }
+      ++n;
+    }
+  }
+  *n_pieces = n;
+  if (n > cap) {
+    set_err("%llu pieces, the list holds %llu", (unsigned long long)n, (unsigned long long)cap);
+    return FR_ERR_CAPACITY;
+  }
+  return FR_OK;
+}
+
 }  // extern "C"

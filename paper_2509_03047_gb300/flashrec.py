@@ -37,6 +37,11 @@ class fr_tensor(ctypes.Structure):
                 ("flags", ctypes.c_uint32)]
 
 
+class fr_piece(ctypes.Structure):
+    _fields_ = [("source", ctypes.c_uint32), ("reserved", ctypes.c_uint32), ("src_off", ctypes.c_uint64),
+                ("dst_off", ctypes.c_uint64), ("nbytes", ctypes.c_uint64)]
+
+
 class FlashrecError(RuntimeError):
     def __init__(self, status: int, where: str):
         self.status = status
@@ -67,6 +72,7 @@ def _load() -> ctypes.CDLL:
     L.fr_unpack_collect.argtypes = [vp, vp, u64, vp, vp]
     L.fr_resend.argtypes = [vp, vp, vp, u64, u64p, vp, vp]
     L.fr_restore.argtypes = [vp, vp, vp, u64, u32, vp, u64, vp, vp, vp]
+    L.fr_shard_pieces.argtypes = [u64, u32, u32, u32, u32, ctypes.POINTER(fr_piece), u64, u64p]
     L.fr_status_str.argtypes = [ctypes.c_int]
     L.fr_status_str.restype = ctypes.c_char_p
     L.fr_last_error.argtypes = []
@@ -75,7 +81,7 @@ def _load() -> ctypes.CDLL:
     for name in ["fr_plan_create", "fr_plan_info", "fr_plan_chunk", "fr_fingerprint", "fr_pack",
                  "fr_unpack_verify", "fr_diff", "fr_sync_status", "fr_version", "fr_fingerprint_static",
                  "fr_plan_create_batched", "fr_plan_batch", "fr_pack_batch", "fr_unpack_verify_batch",
-                 "fr_unpack_collect", "fr_resend", "fr_restore"]:
+                 "fr_unpack_collect", "fr_resend", "fr_restore", "fr_shard_pieces"]:
         getattr(L, name).restype = ctypes.c_int
     return L
 
@@ -255,6 +261,17 @@ def fr_fingerprint_static(tensors: Sequence[torch.Tensor], chunk_bytes: int, out
 
 
 # ---------------------------------------------------------------- convenience
+
+def fr_shard_pieces(n_elems: int, elem_bytes: int, n_dst: int, rank: int, n_src: int):
+    """Pieces of shard `rank` (of `n_dst`) among `n_src` shards of one flat
+    group: a list of (source, src_off, dst_off, nbytes), ascending.  Host only."""
+    n = ctypes.c_uint64(0)
+    cap = max(int(n_src), 1)
+    arr = (fr_piece * cap)()
+    _check(lib.fr_shard_pieces(n_elems, elem_bytes, n_dst, rank, n_src, arr, cap, ctypes.byref(n)),
+           "fr_shard_pieces")
+    return [(arr[i].source, arr[i].src_off, arr[i].dst_off, arr[i].nbytes) for i in range(n.value)]
+
 
 def fp_view(table: torch.Tensor):
     """(crc32c as int64, nonfinite as int64, sumsq as float64) views of a
