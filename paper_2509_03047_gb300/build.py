@@ -38,16 +38,25 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def source_digest() -> str:
-    """Hash of the kernel and ABI sources (identifies what a profile measured)."""
+# Files that define the device kernels (the sweep, finalize, compaction and
+# diff kernels); host-only planning and API code is not among them.
+KERNEL_FILES = ["sweep_fp.cu", "sweep_pack.cu", "sweep_unpack.cu", "finalize.cu", "gf2.cuh", "layout.h", "kernels.h",
+                "sweep_impl.cuh"]
+
+
+def source_digest(kernels_only: bool = False) -> str:
+    """Hash of the sources and compile flags (identifies what a profile
+    measured); with `kernels_only`, of the device-kernel files alone."""
     import hashlib
 
-    h = hashlib.sha256()
-    for name in sorted(SOURCES + HEADERS):
+    h = hashlib.sha256(" ".join(a for a in ARCH + NVCC_FLAGS if not os.path.isabs(a)).encode())
+    names = KERNEL_FILES if kernels_only else SOURCES + HEADERS
+    for name in sorted(names):
         with open(os.path.join(CSRC, name), "rb") as f:
             h.update(name.encode() + b"\0" + f.read())
-    with open(os.path.join(ROOT, "include", "flashrec.h"), "rb") as f:
-        h.update(f.read())
+    if not kernels_only:
+        with open(os.path.join(ROOT, "include", "flashrec.h"), "rb") as f:
+            h.update(f.read())
     return h.hexdigest()[:16]
 
 
