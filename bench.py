@@ -170,7 +170,7 @@ def profiled_traffic(kernel_key: str, workload: str):
     from paper_2509_03047_gb300 import build as _b
 
     ent = rec.get(kernel_key)
-    if not ent or ent.get("workload") != workload or ent.get("sources") != _b.source_digest():
+    if not ent or ent.get("workload") != workload or ent.get("kernel_sources") != _b.source_digest(kernels_only=True):
         return None
     return ent.get("bytes_per_launch")
 
@@ -445,7 +445,10 @@ def run_reference(args):
     if rank != 0:
         return
     cfg = synth.get_config(args.config)
-    idx, tot = sample_buffers(cfg, args.cpu_sample_gb)
+    # size each step's sample so that the W + K steps take about 100 s: the
+    # oracle does one restoration step at roughly 0.1 GB of state per second
+    per_step_s = max(1.0, 100.0 / max(1, args.steps + args.warmup))
+    idx, tot = sample_buffers(cfg, min(args.cpu_sample_gb, 0.1 * per_step_s))
     if cfg.kind == "adam":
         sub = synth.Config(cfg.name, cfg.chunk_bytes, "adam", [cfg.shapes[i // 4] for i in idx[::4]],
                            seed=cfg.seed)
@@ -455,6 +458,8 @@ def run_reference(args):
         state = [torch.randn(specs[i][2] // 4, generator=synth._gen("cpu", cfg.seed, i, 9)) for i in idx]
     host = [t.view(torch.uint8).reshape(-1).numpy() for t in state]
     dts = [FR_DT_BF16 if t.dtype == torch.bfloat16 else FR_DT_F32 for t in state]
+    for _ in range(args.warmup):
+        oracle_sample(cfg, host, dts)
     times = [oracle_sample(cfg, host, dts) for _ in range(args.steps)]
     dt = sum(times) / len(times)
     value = SWEEPS_PER_STEP * tot / dt / 1e9
