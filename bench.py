@@ -309,6 +309,50 @@ def run_flashrec(args):
                 "traffic": profiled_traffic("fr_" + dom, args.config),
                 "alg_bytes_per_launch": alg[dom]}
 
+    # ---- the same step with the fingerprints fused into pack and unpack: the
+    # replica's table comes out of fr_pack_fp, the restored state's out of
+    # fr_unpack_verify_fp, so the step makes two state sweeps instead of four
+    def fused_step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        fr.fr_pack_fp(plan_s.handle, packed, tab_s, stream)
+        if ev:
+            ev[1].record(stream)
+        if flip_idx.numel():
+            packed[flip_idx] ^= flip_mask
+        if ev:
+            ev[2].record(stream)
+        fr.fr_unpack_verify_fp(plan_d.handle, packed, mism, nmis, tab_d, stream)
+        if ev:
+            ev[3].record(stream)
+        fr.fr_diff(tab_s, tab_d, C, div, ndiv, stream)
+        if ev:
+            ev[4].record(stream)
+
+    for _ in range(args.warmup):
+        fused_step()
+    torch.cuda.synchronize()
+    f_mis, f_div = int(nmis.item()), int(ndiv.item())
+    fev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    barrier()
+    torch.cuda.synchronize()
+    for k in range(args.steps):
+        fused_step(fev[k])
+    torch.cuda.synchronize()
+    barrier()
+    f_ms = sum(e[0].elapsed_time(e[4]) for e in fev) / args.steps
+    f_pack = sum(e[0].elapsed_time(e[1]) for e in fev) / args.steps
+    f_unpack = sum(e[2].elapsed_time(e[3]) for e in fev) / args.steps
+    fused = {"ms_per_step": round(f_ms, 3),
+             "state_gbs_4_sweeps_equiv": round(SWEEPS_PER_STEP * S / (f_ms * 1e-3) / 1e9, 1),
+             "pack_fp": {"ms": round(f_pack, 4), "alg_bytes": alg["pack"] + 16 * C,
+                         "frac": round((alg["pack"] + 16 * C) / (f_pack * 1e-3) / 1e9 / peak, 4)},
+             "unpack_verify_fp": {"ms": round(f_unpack, 4), "alg_bytes": alg["unpack_verify"] + 16 * C,
+                                  "frac": round((alg["unpack_verify"] + 16 * C) / (f_unpack * 1e-3) / 1e9 / peak, 4)},
+             "found": {"mismatching_chunks": f_mis, "diverged_chunks": f_div},
+             "how": "fr_pack_fp -> flips -> fr_unpack_verify_fp -> fr_diff: both fingerprint tables come out of "
+                    "the pack and unpack sweeps; same outputs as the step above"}
+
     # ---- end to end through the C ABI with the transfer buffer in pinned host memory
     e2e = None
     if not args.no_e2e:
@@ -321,12 +365,19 @@ def run_flashrec(args):
         s_src, s_dst = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
 
         def restore_step():
+            # both fingerprint tables come out of the restore's own sweeps
+            fr.fr_restore_fp(bs.handle, bd.handle, host_buf, 1, mism, nmis, tab_s, tab_d, s_src, s_dst)
+            fr.fr_diff(tab_s, tab_d, C, div, ndiv, s_dst)
+            s_dst.synchronize()
+            return int(nmis.item()), int(ndiv.item())  # the step's result, read on the host
+
+        def restore_step_unfused():
             fr.fr_fingerprint(bs.handle, tab_s, s_src)
             fr.fr_restore(bs.handle, bd.handle, host_buf, 1, mism, nmis, s_src, s_dst)
             fr.fr_fingerprint(bd.handle, tab_d, s_dst)
             fr.fr_diff(tab_s, tab_d, C, div, ndiv, s_dst)
             s_dst.synchronize()
-            return int(nmis.item()), int(ndiv.item())  # the step's result, read on the host
+            return int(nmis.item()), int(ndiv.item())
 
         restore_step()
         barrier()
@@ -336,7 +387,15 @@ def run_flashrec(args):
             e2e_found = restore_step()
         torch.cuda.synchronize()
         t_e2e = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
-        # (b) for comparison: whole-buffer pack, then whole-buffer unpack
+        # (b) for comparison: the same restore with separate fingerprint sweeps
+        restore_step_unfused()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            restore_step_unfused()
+        torch.cuda.synchronize()
+        t_unfused = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
+        # (c) for comparison: whole-buffer pack, then whole-buffer unpack
         step(buf=host_buf, sync_counts=True)
         torch.cuda.synchronize()
         t0 = time.perf_counter()
@@ -346,8 +405,12 @@ def run_flashrec(args):
         t_serial = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
         e2e = {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_e2e / 1e9, dev), 2), "unit": "GB/s",
                "h2d_bytes_per_step": P, "d2h_bytes_per_step": P + 16, "ms_per_step": round(t_e2e * 1e3, 2),
-               "transfer": "pinned host buffer over NVLink-C2C; fr_restore with %d batches, pack and unpack on "
-                           "two streams, 1 re-send round; no injected flips" % bs.n_batches,
+               "transfer": "pinned host buffer over NVLink-C2C; fr_restore_fp with %d batches, pack and unpack "
+                           "on two streams, both fingerprint tables from the same sweeps, 1 re-send round, then "
+                           "fr_diff; no injected flips" % bs.n_batches,
+               "unfused": {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_unfused / 1e9, dev), 2),
+                           "ms_per_step": round(t_unfused * 1e3, 2),
+                           "how": "fr_fingerprint, fr_restore, fr_fingerprint, fr_diff"},
                "found": {"mismatching_chunks": e2e_found[0], "diverged_chunks": e2e_found[1]},
                "serial": {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_serial / 1e9, dev), 2),
                           "ms_per_step": round(t_serial * 1e3, 2),
@@ -372,7 +435,7 @@ def run_flashrec(args):
                           "l2": "inputs larger than L2 (state %.1f GB vs 129 MB L2); no flush" % (S / 1e9),
                           "parallelism": "replicas only (%d independent rank%s)" % (ws, "s" if ws > 1 else ""),
                           "value_def": "4 sweeps x state bytes / step time"},
-               "calls": calls, "roofline": roofline, "e2e": e2e, "cpu_baseline": cpu,
+               "calls": calls, "roofline": roofline, "fused_step": fused, "e2e": e2e, "cpu_baseline": cpu,
                "gpu_launches": launches_per_step * args.steps, "clocks": clk}
         print(json.dumps(out))
     plan_s.close()

@@ -151,6 +151,39 @@ fr_status fr_unpack_verify(fr_plan plan, const void* src, uint64_t src_bytes,
 fr_status fr_diff(const fr_fp* a_dev, const fr_fp* b_dev, uint64_t n_chunks,
                   uint32_t* diverged_dev, uint64_t cap, uint64_t* n_out_dev, void* stream);
 
+/* ---------------------------------------------------------------- fused fingerprints */
+
+/* A restoration usually wants both fingerprints -- of the replica's state
+ * and of the restored state -- to confirm with fr_diff that they agree.
+ * Pack already computes every fingerprint field of every chunk for its
+ * headers, and unpack reads every restored byte, so these variants also
+ * write the fingerprint table on the same pass, saving the two separate
+ * fr_fingerprint sweeps (half the device traffic of a restore).
+ *
+ * fr_pack_fp: fr_pack, plus `fp_dev` (n_chunks fr_fp entries, 16-byte
+ * aligned, or NULL for none) receives exactly what fr_fingerprint writes for
+ * the plan's tensors.
+ * fr_unpack_verify_fp: fr_unpack_verify, plus `fp_dev` (or NULL) receives the
+ * fingerprint of the restored tensors -- exactly what fr_fingerprint would
+ * write for them afterwards, failing chunks included (their bytes are written
+ * as received).
+ * fr_restore_fp: fr_restore, plus the replica's table in `fp_src_dev` and the
+ * restored state's table in `fp_dst_dev` (either may be NULL); chunks sent
+ * again by a retry get their entries rewritten.  `fp_src_dev` is complete once
+ * `stream_src` reaches the end of the call's work, `fp_dst_dev` once
+ * `stream_dst` does (the call orders the former before the latter).
+ * fr_resend_fp: fr_resend, plus the re-sent chunks' entries rewritten in
+ * `fp_src_dev` and `fp_dst_dev` (either may be NULL).
+ * Errors: as the calls they extend. */
+fr_status fr_pack_fp(fr_plan plan, void* dst, uint64_t dst_bytes, fr_fp* fp_dev, void* stream);
+fr_status fr_unpack_verify_fp(fr_plan plan, const void* src, uint64_t src_bytes, uint32_t* mismatch_dev, uint64_t cap,
+                              uint64_t* n_mismatch_dev, fr_fp* fp_dev, void* stream);
+fr_status fr_restore_fp(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint32_t max_retries,
+                        uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev, fr_fp* fp_src_dev,
+                        fr_fp* fp_dst_dev, void* stream_src, void* stream_dst);
+fr_status fr_resend_fp(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint64_t* n_resent,
+                       fr_fp* fp_src_dev, fr_fp* fp_dst_dev, void* stream_src, void* stream_dst);
+
 /* ---------------------------------------------------------------- streamed restore */
 
 /* The transfer of Sec. III-E end to end: a healthy replica's state reaches a

@@ -16,7 +16,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libflashrec.so")
-SOURCES = ["sweep_fp.cu", "sweep_pack.cu", "sweep_unpack.cu", "finalize.cu", "api.cu", "static_fingerprint.cu"]
+SOURCES = ["sweep_fp.cu", "sweep_pack.cu", "sweep_unpack.cu", "sweep_unpack_fp.cu", "finalize.cu", "api.cu",
+           "static_fingerprint.cu"]
 HEADERS = ["gf2.cuh", "layout.h", "kernels.h", "sweep_impl.cuh"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -40,8 +41,8 @@ def _stale(target: str, deps) -> bool:
 
 # Files that define the device kernels (the sweep, finalize, compaction and
 # diff kernels); host-only planning and API code is not among them.
-KERNEL_FILES = ["sweep_fp.cu", "sweep_pack.cu", "sweep_unpack.cu", "finalize.cu", "gf2.cuh", "layout.h", "kernels.h",
-                "sweep_impl.cuh"]
+KERNEL_FILES = ["sweep_fp.cu", "sweep_pack.cu", "sweep_unpack.cu", "sweep_unpack_fp.cu", "finalize.cu", "gf2.cuh",
+                "layout.h", "kernels.h", "sweep_impl.cuh"]
 
 
 def source_digest(kernels_only: bool = False) -> str:

@@ -110,6 +110,7 @@ fr_status configure_device(int dev) {
   cudaError_t e = configure_sweep_fp();
   if (e == cudaSuccess) e = configure_sweep_pack();
   if (e == cudaSuccess) e = configure_sweep_unpack();
+  if (e == cudaSuccess) e = configure_sweep_unpack_fp();
   if (e != cudaSuccess) return cuda_fail(e, "configure sweep kernels");
   if (dev >= 0 && dev < 64) g_cfg_done |= (1ull << dev);
   return FR_OK;
@@ -271,6 +272,8 @@ fr_status run_batches(fr_plan p, const Decomp& D, int mode, uint8_t* packed, FpE
         e = launch_sweep_fp(sc.dtype, sc.aligned, sp, D.n_ctas, s);
       else if (mode == kModePack)
         e = launch_sweep_pack(sc.dtype, sc.aligned, sp, D.n_ctas, s);
+      else if (mode == kModeUnpackFp)
+        e = launch_sweep_unpack_fp(sc.dtype, sc.aligned, sp, D.n_ctas, s);
       else
         e = launch_sweep_unpack(sc.dtype, sc.aligned, sp, D.n_ctas, s);
       if (e != cudaSuccess) return cuda_fail(e, "sweep kernel launch");
@@ -294,8 +297,10 @@ fr_status run_batches(fr_plan p, const Decomp& D, int mode, uint8_t* packed, FpE
 }
 
 // Sweep + finalize of the `n` chunks listed in `ids` (device), each by one
-// warp: used to re-send chunks that failed verification.
-fr_status run_list(fr_plan p, int mode, const uint32_t* ids, uint64_t n, uint8_t* packed, cudaStream_t s) {
+// warp: used to re-send chunks that failed verification.  `out_fp` (may be
+// null) receives the listed chunks' table entries.
+fr_status run_list(fr_plan p, int mode, const uint32_t* ids, uint64_t n, uint8_t* packed, FpEntry* out_fp,
+                   cudaStream_t s) {
   if (n == 0) return FR_OK;
   ListParams lp;
   lp.chunks = p->whole.d_chunks;
@@ -316,7 +321,7 @@ fr_status run_list(fr_plan p, int mode, const uint32_t* ids, uint64_t n, uint8_t
   fp.c_end = n;
   fp.ids = ids;
   fp.packed = packed;
-  fp.out_fp = nullptr;
+  fp.out_fp = out_fp;
   fp.flags = p->d_flags;
   e = launch_finalize(mode, fp, s);
   if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
@@ -357,9 +362,10 @@ fr_status check_same_layout(fr_plan src, fr_plan dst) {
 
 // One re-send: list the chunks whose last verdict in `dst` failed (a host
 // sync learns how many), re-pack them from `src` on `ss`, and re-unpack them
-// on `sd` after that.  *failing gets the number re-sent.
+// on `sd` after that.  *failing gets the number re-sent.  Non-null fp_src /
+// fp_dst get the re-sent chunks' table entries on either side.
 fr_status resend_failed(fr_plan src, fr_plan dst, uint8_t* buf, cudaStream_t ss, cudaStream_t sd,
-                        uint64_t* failing) {
+                        uint64_t* failing, FpEntry* fp_src = nullptr, FpEntry* fp_dst = nullptr) {
   *failing = 0;
   cudaError_t e =
       launch_compact_flags(dst->d_flags, dst->n_chunks, dst->d_ids, dst->n_chunks, dst->d_count, nullptr, sd);
@@ -372,11 +378,11 @@ fr_status resend_failed(fr_plan src, fr_plan dst, uint8_t* buf, cudaStream_t ss,
   cudaEvent_t ev_ids = dst->events[dst->n_batches], ev_packed = src->events[src->n_batches];
   if ((e = cudaEventRecord(ev_ids, sd)) != cudaSuccess || (e = cudaStreamWaitEvent(ss, ev_ids, 0)) != cudaSuccess)
     return cuda_fail(e, "order the re-send");
-  fr_status st = run_list(src, kModePack, dst->d_ids, n, buf, ss);
+  fr_status st = run_list(src, kModePack, dst->d_ids, n, buf, fp_src, ss);
   if (st != FR_OK) return st;
   if ((e = cudaEventRecord(ev_packed, ss)) != cudaSuccess || (e = cudaStreamWaitEvent(sd, ev_packed, 0)) != cudaSuccess)
     return cuda_fail(e, "order the re-send");
-  st = run_list(dst, kModeUnpack, dst->d_ids, n, buf, sd);
+  st = run_list(dst, fp_dst ? kModeUnpackFp : kModeUnpack, dst->d_ids, n, buf, fp_dst, sd);
   if (st != FR_OK) return st;
   *failing = n;
   return FR_OK;
@@ -569,18 +575,27 @@ fr_status fr_fingerprint(fr_plan p, fr_fp* out_dev, void* stream) {
 }
 
 fr_status fr_pack(fr_plan p, void* dst, uint64_t dst_bytes, void* stream) {
+  return fr_pack_fp(p, dst, dst_bytes, nullptr, stream);
+}
+
+fr_status fr_pack_fp(fr_plan p, void* dst, uint64_t dst_bytes, fr_fp* fp_dev, void* stream) {
   if (p == nullptr) return invalid("plan is null");
   if (p->n_chunks == 0) return FR_OK;
   fr_status st = check_packed_buffer(p, dst, dst_bytes);
   if (st != FR_OK) return st;
   DeviceGuard g(p->device);
   if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
-  return run_batches(p, p->whole, kModePack, static_cast<uint8_t*>(dst), nullptr, 0, 1,
+  return run_batches(p, p->whole, kModePack, static_cast<uint8_t*>(dst), reinterpret_cast<FpEntry*>(fp_dev), 0, 1,
                      static_cast<cudaStream_t>(stream));
 }
 
 fr_status fr_unpack_verify(fr_plan p, const void* src, uint64_t src_bytes, uint32_t* mismatch_dev, uint64_t cap,
                            uint64_t* n_mismatch_dev, void* stream) {
+  return fr_unpack_verify_fp(p, src, src_bytes, mismatch_dev, cap, n_mismatch_dev, nullptr, stream);
+}
+
+fr_status fr_unpack_verify_fp(fr_plan p, const void* src, uint64_t src_bytes, uint32_t* mismatch_dev, uint64_t cap,
+                              uint64_t* n_mismatch_dev, fr_fp* fp_dev, void* stream) {
   if (p == nullptr) return invalid("plan is null");
   if (n_mismatch_dev == nullptr) return invalid("n_mismatch_dev is null");
   if (cap > 0 && mismatch_dev == nullptr) return invalid("mismatch_dev is null");
@@ -593,7 +608,8 @@ fr_status fr_unpack_verify(fr_plan p, const void* src, uint64_t src_bytes, uint3
   }
   fr_status st = check_packed_buffer(p, src, src_bytes);
   if (st != FR_OK) return st;
-  st = run_batches(p, p->whole, kModeUnpack, const_cast<uint8_t*>(static_cast<const uint8_t*>(src)), nullptr, 0, 1, s);
+  st = run_batches(p, p->whole, fp_dev ? kModeUnpackFp : kModeUnpack,
+                   const_cast<uint8_t*>(static_cast<const uint8_t*>(src)), reinterpret_cast<FpEntry*>(fp_dev), 0, 1, s);
   if (st != FR_OK) return st;
   cudaError_t e = launch_compact_flags(p->d_flags, p->n_chunks, mismatch_dev, cap, n_mismatch_dev, p->d_status, s);
   return e == cudaSuccess ? FR_OK : cuda_fail(e, "compaction kernel launch");
@@ -642,6 +658,13 @@ fr_status fr_unpack_collect(fr_plan p, uint32_t* mismatch_dev, uint64_t cap, uin
 fr_status fr_restore(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint32_t max_retries,
                      uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev, void* stream_src,
                      void* stream_dst) {
+  return fr_restore_fp(src, dst, staging, staging_bytes, max_retries, mismatch_dev, cap, n_mismatch_dev, nullptr,
+                       nullptr, stream_src, stream_dst);
+}
+
+fr_status fr_restore_fp(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint32_t max_retries,
+                        uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev, fr_fp* fp_src_dev,
+                        fr_fp* fp_dst_dev, void* stream_src, void* stream_dst) {
   if (src == nullptr || dst == nullptr) return invalid("plan is null");
   if (n_mismatch_dev == nullptr) return invalid("n_mismatch_dev is null");
   if (cap > 0 && mismatch_dev == nullptr) return invalid("mismatch_dev is null");
@@ -659,21 +682,23 @@ fr_status fr_restore(fr_plan src, fr_plan dst, void* staging, uint64_t staging_b
   uint8_t* buf = static_cast<uint8_t*>(staging);
   const Decomp& DS = batch_decomp(src);
   const Decomp& DD = batch_decomp(dst);
+  FpEntry* fs = reinterpret_cast<FpEntry*>(fp_src_dev);
+  FpEntry* fd = reinterpret_cast<FpEntry*>(fp_dst_dev);
   cudaError_t e;
   // Pipeline: batch b is unpacked on the receiver's stream as soon as the
   // replica's stream has packed it, while the replica packs batch b+1.
   for (uint32_t b = 0; b < src->n_batches; ++b) {
-    st = run_batches(src, DS, kModePack, buf, nullptr, b, b + 1, ss);
+    st = run_batches(src, DS, kModePack, buf, fs, b, b + 1, ss);
     if (st != FR_OK) return st;
     if ((e = cudaEventRecord(src->events[b], ss)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
     if ((e = cudaStreamWaitEvent(sd, src->events[b], 0)) != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
-    st = run_batches(dst, DD, kModeUnpack, buf, nullptr, b, b + 1, sd);
+    st = run_batches(dst, DD, fd ? kModeUnpackFp : kModeUnpack, buf, fd, b, b + 1, sd);
     if (st != FR_OK) return st;
   }
   // Retries: re-send only the chunks that failed, straight from the replica.
   for (uint32_t r = 0; r < max_retries; ++r) {
     uint64_t failing = 0;
-    st = resend_failed(src, dst, buf, ss, sd, &failing);
+    st = resend_failed(src, dst, buf, ss, sd, &failing, fs, fd);
     if (st != FR_OK) return st;
     if (failing == 0) break;
   }
@@ -688,6 +713,11 @@ fr_status fr_restore(fr_plan src, fr_plan dst, void* staging, uint64_t staging_b
 
 fr_status fr_resend(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint64_t* n_resent,
                     void* stream_src, void* stream_dst) {
+  return fr_resend_fp(src, dst, staging, staging_bytes, n_resent, nullptr, nullptr, stream_src, stream_dst);
+}
+
+fr_status fr_resend_fp(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint64_t* n_resent,
+                       fr_fp* fp_src_dev, fr_fp* fp_dst_dev, void* stream_src, void* stream_dst) {
   if (src == nullptr || dst == nullptr) return invalid("plan is null");
   fr_status st = check_same_layout(src, dst);
   if (st != FR_OK) return st;
@@ -699,7 +729,8 @@ fr_status fr_resend(fr_plan src, fr_plan dst, void* staging, uint64_t staging_by
   if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
   uint64_t n = 0;
   st = resend_failed(src, dst, static_cast<uint8_t*>(staging), static_cast<cudaStream_t>(stream_src),
-                     static_cast<cudaStream_t>(stream_dst), &n);
+                     static_cast<cudaStream_t>(stream_dst), &n, reinterpret_cast<FpEntry*>(fp_src_dev),
+                     reinterpret_cast<FpEntry*>(fp_dst_dev));
   if (n_resent) *n_resent = n;
   return st;
 }

@@ -16,6 +16,7 @@
 //      the zero padding after the payload and, for the last chunk, the zero gap
 //      after the header table; unpack: checks the header against the plan, the
 //      header CRC, the payload CRC and the padding, and writes a verdict.
+//      Pack and unpack-fp also write the table entry when given a table.
 // The verdicts become an ascending id list through a single-CTA ordered
 // compaction, which fr_diff shares with a different predicate.
 #include <cuda_runtime.h>
@@ -97,7 +98,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
     const ChunkDesc cd = p.chunks[c];
     const uint64_t body = cd.len & ~static_cast<uint64_t>(kBlockBytes - 1);
     const uint32_t tail = static_cast<uint32_t>(cd.len - body);
-    const bool values = (MODE != kModeUnpack) && (cd.dtype != kDtBytes);
+    const bool values = mode_sums(MODE) && (cd.dtype != kDtBytes);
     // list mode: one record per chunk with a body, at the list position
     const uint64_t first_rec = p.ids ? pos : cd.first_rec;
     const int64_t n_recs = p.ids ? (body ? 1 : 0) : cd.n_recs;
@@ -135,7 +136,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
     if (values) {
       const uint64_t n_seg = (body / kBlockBytes + kSegBlocks - 1) / kSegBlocks;
       double s = 0.0;
-      for (uint64_t k = lane; k < n_seg; k += 32) s += p.segs[cd.seg_base + k];
+      for (uint64_t k = lane; k < n_seg; k += 32) s += seg_value(p.segs + cd.seg_base + k);
 #pragma unroll
       for (int m = 16; m >= 1; m >>= 1) s += __shfl_down_sync(kFull, s, m);
       sq_rec = s;
@@ -144,7 +145,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
     // ---- 2. tail
     const uint8_t* tsrc;
     uint8_t* tdst = nullptr;
-    if (MODE == kModeUnpack) {
+    if (mode_unpacks(MODE)) {
       tsrc = p.packed + cd.payload_off + body;
       tdst = reinterpret_cast<uint8_t*>(cd.addr) + body;
     } else {
@@ -193,7 +194,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
     const bool last = (c + 1 == p.n_chunks);
 
     // ---- 4. outputs
-    if (MODE == kModeFingerprint) {
+    if (MODE != kModeUnpack && p.out_fp != nullptr) {  // the fingerprint table (optional for pack, unpack-fp)
       if (lane == 0) {
         FpEntry e;
         e.crc32c = crc;
@@ -201,7 +202,8 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
         e.sumsq = sumsq;
         p.out_fp[c] = e;
       }
-    } else if (MODE == kModePack) {
+    }
+    if (MODE == kModePack) {
       if (lane == 0) {
         uint32_t h[16];
         const uint64_t sbits = static_cast<uint64_t>(__double_as_longlong(sumsq));
@@ -231,7 +233,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
       if (last)
         for (uint64_t j = table_end + lane * 16u; j < gap_end; j += 512)
           *reinterpret_cast<uint4*>(p.packed + j) = make_uint4(0, 0, 0, 0);
-    } else {  // unpack + verify
+    } else if (mode_unpacks(MODE)) {  // unpack + verify
       bool bad = false;
       if (lane == 0) {
         const uint4* src = reinterpret_cast<const uint4*>(p.packed + c * kHeaderBytes);
@@ -350,6 +352,8 @@ cudaError_t launch_finalize(int mode, const FinalizeParams& p, cudaStream_t s) {
     finalize_kernel<kModeFingerprint><<<grid, kFinThreads, 0, s>>>(p);
   else if (mode == kModePack)
     finalize_kernel<kModePack><<<grid, kFinThreads, 0, s>>>(p);
+  else if (mode == kModeUnpackFp)
+    finalize_kernel<kModeUnpackFp><<<grid, kFinThreads, 0, s>>>(p);
   else
     finalize_kernel<kModeUnpack><<<grid, kFinThreads, 0, s>>>(p);
   return cudaGetLastError();

@@ -9,14 +9,21 @@
 
 namespace frk {
 
-enum : int { kModeFingerprint = 0, kModePack = 1, kModeUnpack = 2 };
+// Sweep modes.  kModeUnpackFp is unpack + verify that also computes the
+// fingerprint values (non-finite count, sum of squares) of the restored bytes
+// on the same pass, so a restore needs no separate fingerprint sweep.
+enum : int { kModeFingerprint = 0, kModePack = 1, kModeUnpack = 2, kModeUnpackFp = 3 };
+// Direction: the packed buffer is the source.
+__host__ __device__ constexpr bool mode_unpacks(int m) { return m == kModeUnpack || m == kModeUnpackFp; }
+// Whether the mode computes non-finite counts and sums of squares.
+__host__ __device__ constexpr bool mode_sums(int m) { return m != kModeUnpack; }
 
 struct SweepParams {
   const ChunkDesc* chunks;
   const WarpDesc* warps;  // this class's per-warp ranges
   const uint32_t* class_chunks;  // ids of this class's chunks with a body, in order
   Record* recs;
-  double* segs;           // segment sums of squares (fingerprint, pack)
+  double* segs;           // segment sums of squares (all modes but kModeUnpack)
   uint8_t* packed;        // pack: destination; unpack: source; fingerprint: unused
   uint32_t n_warps;       // warps with a descriptor
 };
@@ -30,7 +37,7 @@ struct FinalizeParams {
   uint64_t c_begin, c_end;  // chunks to finalize: [c_begin, c_end), or list positions if ids != null
   const uint32_t* ids;      // list mode: chunk ids; the record of list position i is recs[i]
   uint8_t* packed;  // pack: destination; unpack: source
-  FpEntry* out_fp;  // fingerprint: output table
+  FpEntry* out_fp;  // fingerprint: output table; pack, unpack-fp: optional table (null: none)
   uint8_t* flags;   // unpack: per-chunk verdict
 };
 
@@ -45,6 +52,7 @@ constexpr int kSweepWarps = FR_SWEEP_WARPS;
 cudaError_t configure_sweep_fp();
 cudaError_t configure_sweep_pack();
 cudaError_t configure_sweep_unpack();
+cudaError_t configure_sweep_unpack_fp();
 
 // List mode: one warp per listed chunk sweeps its whole body into recs[i].
 struct ListParams {
@@ -61,9 +69,12 @@ cudaError_t launch_sweep_fp(uint32_t dtype, bool aligned, const SweepParams& p, 
 cudaError_t launch_sweep_pack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
 cudaError_t launch_sweep_unpack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
 cudaError_t launch_list_pack(const ListParams& p, cudaStream_t s);
+cudaError_t launch_sweep_unpack_fp(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
 cudaError_t launch_list_unpack(const ListParams& p, cudaStream_t s);
+cudaError_t launch_list_unpack_fp(const ListParams& p, cudaStream_t s);
 inline cudaError_t launch_list_sweep(int mode, const ListParams& p, cudaStream_t s) {
-  return mode == kModePack ? launch_list_pack(p, s) : launch_list_unpack(p, s);
+  return mode == kModePack ? launch_list_pack(p, s)
+                           : (mode == kModeUnpackFp ? launch_list_unpack_fp(p, s) : launch_list_unpack(p, s));
 }
 
 cudaError_t launch_finalize(int mode, const FinalizeParams& p, cudaStream_t s);

@@ -28,6 +28,24 @@ constexpr uint64_t kHeaderBytes = 64;
 #endif
 constexpr uint64_t kSegBlocks = FR_SEG_BLOCKS;
 static_assert((kSegBlocks & (kSegBlocks - 1)) == 0, "a power of two");
+// A segment's 8-byte slot holds its sum in one of two forms, told apart by
+// bit 63:
+//   clear: an unevaluated float pair, lo in bytes 0-3 and hi (>= +0) in
+//          bytes 4-7, whose exact sum is the segment's sum to about 2^-44
+//          relative -- the common case, which keeps the sweep off the narrow
+//          fp64 pipe;
+//   set:   the sum as a double, negated (sums are >= 0, so -0.0 for zero) --
+//          segments that needed the exact element-by-element path, or whose
+//          sum is too large for the float form.
+// seg_value() reads either form as a double.
+#ifdef __CUDACC__
+__host__ __device__
+#endif
+inline double seg_value(const double* slot) {
+  if (*reinterpret_cast<const uint64_t*>(slot) >> 63) return -*slot;
+  const float* f = reinterpret_cast<const float*>(slot);
+  return static_cast<double>(f[1]) + static_cast<double>(f[0]);
+}
 constexpr uint64_t kPayloadAlign = 256;
 constexpr uint32_t kMagic = 0x31435246u;  // bytes 'F','R','C','1'
 constexpr uint32_t kVersion = 1;

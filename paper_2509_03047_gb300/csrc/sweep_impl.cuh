@@ -302,19 +302,19 @@ __device__ __noinline__ bool span_is_zero(const uint8_t* sp, uint64_t b0, uint64
   return acc == 0;
 }
 
-// The span's sum as a double.  The four fp32 partial sums are first merged
-// error-free in fp32 (TwoSum), so only two conversions and one fp64 add reach
-// the narrow fp64 pipe; the error terms (about 2^-24 of the sum) are merged
-// with plain fp32 adds, which costs about 2^-48 relative.
-__device__ __forceinline__ double fold_to_double(const FpAcc& f) {
+// The span's sum as an unevaluated float pair (hi, lo): the four fp32 partial
+// sums are merged error-free in fp32 (TwoSum); the error terms (about 2^-24
+// of the sum) are merged with plain fp32 adds, which costs about 2^-48
+// relative.  No fp64 work: GB300's fp64 pipe is narrow.
+__device__ __forceinline__ void fold_to_pair(const FpAcc& f, float& hi, float& lo) {
   u64 s = f.A, c = add2(f.CA, f.CB);
-  two_sum_acc(s, c, f.B);  // s + c == A + B + CA + CB up to the rounding of c
+  two_sum_acc(s, c, f.B);
   const float a = lo_f(s), b = hi_f(s);
-  const float t = a + b;  // scalar TwoSum of the two halves
+  const float t = a + b;
   const float z = t - a;
   const float err = (a - (t - z)) + (b - z);
-  const float lo = (lo_f(c) + hi_f(c)) + err;
-  return static_cast<double>(t) + static_cast<double>(lo);
+  hi = t;
+  lo = (lo_f(c) + hi_f(c)) + err;
 }
 
 // ------------------------------------------------------------------ piece
@@ -327,15 +327,18 @@ __device__ __forceinline__ void prefetch_l2(const uint8_t* p, uint32_t bytes) {
 // Per-mode pipeline geometry: blocks per lane held in registers one stage
 // ahead, and spans (kSpan blocks) prefetched into L2 ahead of use.
 template <int MODE>
+// Unpack with fingerprint values does pack's work per byte (copy, CRC, sums),
+// so it takes pack's geometry.
 struct Geo {
-  static constexpr int kStage = MODE == kModeFingerprint ? FR_STAGE_FP : (MODE == kModePack ? FR_STAGE_PACK
-                                                                                              : FR_STAGE_UNPACK);
-  static constexpr int kAhead = MODE == kModeFingerprint ? FR_AHEAD_FP : (MODE == kModePack ? FR_AHEAD_PACK
-                                                                                              : FR_AHEAD_UNPACK);
+  static constexpr bool kPackLike = MODE == kModePack || MODE == kModeUnpackFp;
+  static constexpr int kStage = MODE == kModeFingerprint ? FR_STAGE_FP : (kPackLike ? FR_STAGE_PACK
+                                                                                    : FR_STAGE_UNPACK);
+  static constexpr int kAhead = MODE == kModeFingerprint ? FR_AHEAD_FP : (kPackLike ? FR_AHEAD_PACK
+                                                                                    : FR_AHEAD_UNPACK);
   // Issue a unit's reload before consuming it (more load lead, one register
   // copy) or after (no copy): latency-bound modes want the former.
   static constexpr bool kLoadFirst = MODE == kModeFingerprint ? FR_LOADFIRST_FP
-                                     : (MODE == kModePack ? FR_LOADFIRST_PACK : FR_LOADFIRST_UNPACK);
+                                     : (kPackLike ? FR_LOADFIRST_PACK : FR_LOADFIRST_UNPACK);
   static_assert(kSpan % kStage == 0, "a span holds whole stages");
 };
 
@@ -349,7 +352,7 @@ struct Lane {
 
 template <int MODE, int DT, int DAL>
 __device__ __forceinline__ void do_unit(Lane<MODE, DT>& L, const uint4& v, uint8_t* wp, uint32_t lb) {
-  constexpr bool kFp = (MODE != kModeUnpack) && (DT != kDtBytes);
+  constexpr bool kFp = mode_sums(MODE) && (DT != kDtBytes);
   if (MODE != kModeFingerprint) st_unit<DAL>(wp, v);
   L.s[0] = braid_step(L.s[0] ^ v.x, lb);
   L.s[1] = braid_step(L.s[1] ^ v.y, lb);
@@ -362,7 +365,7 @@ __device__ __forceinline__ void do_unit(Lane<MODE, DT>& L, const uint4& v, uint8
 // either large enough that fp32 underflow is negligible (below 2^-77 relative)
 // or made of zeros only; otherwise the segment is summed exactly from a
 // reload.  The lanes' sums are then added in a fixed tree and lane 0 stores
-// the segment's sum at its index.
+// the segment's sum (a float pair, see seg_value) at its index.
 template <int MODE, int DT, int SAL>
 __device__ __forceinline__ void span_end(Lane<MODE, DT>& L, const uint8_t* sp, uint64_t b0, uint64_t b1,
                                          double* seg, uint32_t lane) {
@@ -370,18 +373,37 @@ __device__ __forceinline__ void span_end(Lane<MODE, DT>& L, const uint8_t* sp, u
   const float tot = lo_f(ab) + hi_f(ab);
   bool ok = tot < __int_as_float(0x7F800000);
   if (ok && !(tot >= 0x1p-60f)) ok = span_is_zero<DT, SAL>(sp, b0, b1);
-  double d;
+  float hi = 0.0f, lo = 0.0f;
+  double d = 0.0;
   if (ok) {
-    d = fold_to_double(L.f);
+    fold_to_pair(L.f, hi, lo);
   } else {
     const Exact x = slow_span<DT, SAL>(sp, b0, b1);
     d = x.d;
     L.nonfinite += x.nonfinite;
   }
   L.f.A = L.f.CA = L.f.B = L.f.CB = 0ull;
+  // The lanes' sums are added in a fixed tree: as float pairs by TwoSum when
+  // every lane took the fast path with a sum far from fp32 overflow (no fp64
+  // work), else in fp64 (rare).  Lane 0 stores the form seg_value() reads.
+  if (__all_sync(0xFFFFFFFFu, ok && tot < 0x1p120f)) {
 #pragma unroll
-  for (int m = 16; m >= 1; m >>= 1) d += __shfl_down_sync(0xFFFFFFFFu, d, m);
-  if (lane == 0) *seg = d;
+    for (int m = 16; m >= 1; m >>= 1) {
+      const float oh = __shfl_down_sync(0xFFFFFFFFu, hi, m);
+      const float ol = __shfl_down_sync(0xFFFFFFFFu, lo, m);
+      const float t = hi + oh;
+      const float z = t - hi;
+      const float err = (hi - (t - z)) + (oh - z);
+      lo = (lo + ol) + err;
+      hi = t;
+    }
+    if (lane == 0) *reinterpret_cast<float2*>(seg) = make_float2(lo, hi);
+  } else {
+    if (ok) d = static_cast<double>(hi) + static_cast<double>(lo);
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) d += __shfl_down_sync(0xFFFFFFFFu, d, m);
+    if (lane == 0) *seg = -d;
+  }
 }
 
 // One piece: `nblk` 512-byte blocks from `src` (to `dst` for pack/unpack).
@@ -395,7 +417,7 @@ __device__ __forceinline__ void span_end(Lane<MODE, DT>& L, const uint8_t* sp, u
 template <int MODE, int DT, int SAL, int DAL>
 __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
                                             uint64_t nblk, uint32_t lane, Record* rec, double* segs) {
-  constexpr bool kFp = (MODE != kModeUnpack) && (DT != kDtBytes);
+  constexpr bool kFp = mode_sums(MODE) && (DT != kDtBytes);
   constexpr int kStage = Geo<MODE>::kStage;
   constexpr int kAhead = Geo<MODE>::kAhead;
   constexpr uint32_t kStageBytes = kStage * kBlockBytes;
@@ -500,7 +522,7 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
 template <int MODE, int DT, int AL>
 __device__ __forceinline__ void sweep_piece_al(const uint8_t* tensor, uint8_t* packed, uint64_t n,
                                                uint32_t lane, Record* rec, double* segs) {
-  if (MODE == kModeUnpack)
+  if (mode_unpacks(MODE))
     sweep_piece<MODE, DT, 16, AL>(packed, const_cast<uint8_t*>(tensor), n, lane, rec, segs);
   else
     sweep_piece<MODE, DT, AL, 16>(tensor, packed, n, lane, rec, segs);
@@ -568,7 +590,7 @@ __global__ void __launch_bounds__(kThreads, 1) list_kernel(ListParams p) {
   const uint8_t* tensor = reinterpret_cast<const uint8_t*>(cd.addr);
   uint8_t* packed = (MODE == kModeFingerprint) ? nullptr : p.packed + cd.payload_off;
   const bool aligned = (cd.sweep_class & 1u) != 0;
-  const uint32_t dt = (MODE == kModeUnpack) ? kDtBytes : cd.dtype;
+  const uint32_t dt = mode_sums(MODE) ? cd.dtype : kDtBytes;
   double* segs = p.segs + cd.seg_base;
   Record* rec = p.recs + w;
   if (dt == kDtF32) {
@@ -605,14 +627,14 @@ cudaError_t launch_one(const SweepParams& p, int n_ctas, cudaStream_t s) {
 
 }  // namespace
 
-// Configure / launch every class kernel of one mode (unpack ignores the
+// Configure / launch every class kernel of one mode (plain unpack ignores the
 // element type: it only checksums and copies).
 template <int MODE>
 cudaError_t configure_mode() {
   cudaError_t e = cudaFuncSetAttribute(list_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTableBytes);
   if (e == cudaSuccess) e = configure_one<MODE, kDtBytes, true>();
   if (e == cudaSuccess) e = configure_one<MODE, kDtBytes, false>();
-  if (MODE != kModeUnpack) {
+  if (mode_sums(MODE)) {
     if (e == cudaSuccess) e = configure_one<MODE, kDtBf16, true>();
     if (e == cudaSuccess) e = configure_one<MODE, kDtBf16, false>();
     if (e == cudaSuccess) e = configure_one<MODE, kDtF32, true>();
@@ -623,7 +645,7 @@ cudaError_t configure_mode() {
 
 template <int MODE>
 cudaError_t launch_mode(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s) {
-  if (MODE == kModeUnpack || dtype == kDtBytes)
+  if (!mode_sums(MODE) || dtype == kDtBytes)
     return aligned ? launch_one<MODE, kDtBytes, true>(p, n_ctas, s) : launch_one<MODE, kDtBytes, false>(p, n_ctas, s);
   if (dtype == kDtBf16)
     return aligned ? launch_one<MODE, kDtBf16, true>(p, n_ctas, s) : launch_one<MODE, kDtBf16, false>(p, n_ctas, s);

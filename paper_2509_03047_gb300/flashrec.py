@@ -73,6 +73,10 @@ def _load() -> ctypes.CDLL:
     L.fr_resend.argtypes = [vp, vp, vp, u64, u64p, vp, vp]
     L.fr_restore.argtypes = [vp, vp, vp, u64, u32, vp, u64, vp, vp, vp]
     L.fr_shard_pieces.argtypes = [u64, u32, u32, u32, u32, ctypes.POINTER(fr_piece), u64, u64p]
+    L.fr_pack_fp.argtypes = [vp, vp, u64, vp, vp]
+    L.fr_unpack_verify_fp.argtypes = [vp, vp, u64, vp, u64, vp, vp, vp]
+    L.fr_restore_fp.argtypes = [vp, vp, vp, u64, u32, vp, u64, vp, vp, vp, vp, vp]
+    L.fr_resend_fp.argtypes = [vp, vp, vp, u64, u64p, vp, vp, vp, vp]
     L.fr_status_str.argtypes = [ctypes.c_int]
     L.fr_status_str.restype = ctypes.c_char_p
     L.fr_last_error.argtypes = []
@@ -81,7 +85,8 @@ def _load() -> ctypes.CDLL:
     for name in ["fr_plan_create", "fr_plan_info", "fr_plan_chunk", "fr_fingerprint", "fr_pack",
                  "fr_unpack_verify", "fr_diff", "fr_sync_status", "fr_version", "fr_fingerprint_static",
                  "fr_plan_create_batched", "fr_plan_batch", "fr_pack_batch", "fr_unpack_verify_batch",
-                 "fr_unpack_collect", "fr_resend", "fr_restore", "fr_shard_pieces"]:
+                 "fr_unpack_collect", "fr_resend", "fr_restore", "fr_shard_pieces", "fr_pack_fp", "fr_unpack_verify_fp",
+                 "fr_restore_fp", "fr_resend_fp"]:
         getattr(L, name).restype = ctypes.c_int
     return L
 
@@ -188,6 +193,46 @@ def fr_restore(src_plan, dst_plan, staging: torch.Tensor, max_retries: int, mism
     _check(lib.fr_restore(src_plan, dst_plan, staging.data_ptr() if staging.numel() else None, staging.numel(),
                           max_retries, mismatch.data_ptr() if cap else None, cap, count.data_ptr(),
                           _stream(stream_src), _stream(stream_dst)), "fr_restore")
+
+
+def _table_ptr(t: Optional[torch.Tensor]):
+    return None if t is None else t.data_ptr()
+
+
+def fr_pack_fp(plan, dst: torch.Tensor, fp: Optional[torch.Tensor], stream=None) -> None:
+    """fr_pack that also writes the fingerprint table `fp` (uint8, 16 B per chunk)."""
+    _check(lib.fr_pack_fp(plan, dst.data_ptr() if dst.numel() else None, dst.numel() * dst.element_size(),
+                          _table_ptr(fp), _stream(stream)), "fr_pack_fp")
+
+
+def fr_unpack_verify_fp(plan, src: torch.Tensor, mismatch: Optional[torch.Tensor], count: torch.Tensor,
+                        fp: Optional[torch.Tensor], stream=None) -> None:
+    """fr_unpack_verify that also writes the restored tensors' fingerprint table."""
+    cap = 0 if mismatch is None else mismatch.numel()
+    _check(lib.fr_unpack_verify_fp(plan, src.data_ptr() if src.numel() else None, src.numel() * src.element_size(),
+                                   mismatch.data_ptr() if cap else None, cap, count.data_ptr(), _table_ptr(fp),
+                                   _stream(stream)), "fr_unpack_verify_fp")
+
+
+def fr_restore_fp(src_plan, dst_plan, staging: torch.Tensor, max_retries: int, mismatch: Optional[torch.Tensor],
+                  count: torch.Tensor, fp_src: Optional[torch.Tensor], fp_dst: Optional[torch.Tensor],
+                  stream_src=None, stream_dst=None) -> None:
+    """fr_restore that also writes both fingerprint tables."""
+    cap = 0 if mismatch is None else mismatch.numel()
+    _check(lib.fr_restore_fp(src_plan, dst_plan, staging.data_ptr() if staging.numel() else None, staging.numel(),
+                             max_retries, mismatch.data_ptr() if cap else None, cap, count.data_ptr(),
+                             _table_ptr(fp_src), _table_ptr(fp_dst), _stream(stream_src), _stream(stream_dst)),
+           "fr_restore_fp")
+
+
+def fr_resend_fp(src_plan, dst_plan, staging: torch.Tensor, fp_src: Optional[torch.Tensor],
+                 fp_dst: Optional[torch.Tensor], stream_src=None, stream_dst=None) -> int:
+    """fr_resend that also rewrites the re-sent chunks' fingerprint entries."""
+    n = ctypes.c_uint64()
+    _check(lib.fr_resend_fp(src_plan, dst_plan, staging.data_ptr() if staging.numel() else None, staging.numel(),
+                            ctypes.byref(n), _table_ptr(fp_src), _table_ptr(fp_dst), _stream(stream_src),
+                            _stream(stream_dst)), "fr_resend_fp")
+    return n.value
 
 
 def fr_plan_info(plan):

@@ -107,6 +107,8 @@ def test_special_values():
         torch.full((n,), 1e-25, device="cuda"),             # squares underflow fp32
         torch.full((n,), 3e19, device="cuda"),              # squares overflow fp32
         torch.full((n,), 3.0e38, device="cuda"),
+        torch.full((n,), 1e17, device="cuda"),              # segment sums near fp32's top, fast path
+        torch.full((n,), 2e17, device="cuda"),              # lane sums above 2^120: fp64 tree
         torch.full((n,), float("nan"), device="cuda"),
         torch.full((n,), float("inf"), device="cuda"),
         torch.full((n,), 0.5, device="cuda"),
@@ -127,7 +129,7 @@ def test_special_values():
     t = table_np(got["table"])
     per = (n * 4) // (16 * KiB)
     assert (t["sumsq"][:per] == 0).all()
-    assert (t["nonfinite"][6 * per:8 * per] == (16 * KiB) // 4).all()
+    assert (t["nonfinite"][8 * per:10 * per] == (16 * KiB) // 4).all()
 
 
 def test_many_tiny_tensors():
