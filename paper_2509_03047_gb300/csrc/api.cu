@@ -55,6 +55,7 @@ struct Decomp {
   WarpDesc* d_warps = nullptr;
   uint32_t* d_lists = nullptr;
   uint64_t* d_rec_nblk = nullptr;
+  uint32_t* d_rec_mul = nullptr;  // per record: x^(8 * bytes after it in its chunk)
   Record* d_recs = nullptr;
 };
 
@@ -70,6 +71,7 @@ struct fr_plan_s {
   Decomp batched;                 // n_batches > 1: batches over half the SMs
   uint64_t n_segs = 0;            // 16 KiB sum segments of all chunk bodies
   double* d_segs = nullptr;       // their sums of squares
+  uint32_t* d_crc_xor = nullptr;  // per chunk: the CRC preset/final-XOR term of its length
   uint8_t* d_flags = nullptr;     // unpack verdict per chunk
   uint32_t* d_status = nullptr;
   uint32_t* d_ids = nullptr;      // restore: ids of failing chunks (capacity n_chunks)
@@ -147,6 +149,7 @@ void free_decomp(Decomp& D) {
   cudaFree(D.d_warps);
   cudaFree(D.d_lists);
   cudaFree(D.d_rec_nblk);
+  cudaFree(D.d_rec_mul);
   cudaFree(D.d_recs);
   D = Decomp();
 }
@@ -155,6 +158,7 @@ void free_device(fr_plan p) {
   free_decomp(p->whole);
   free_decomp(p->batched);
   cudaFree(p->d_segs);
+  cudaFree(p->d_crc_xor);
   cudaFree(p->d_flags);
   cudaFree(p->d_status);
   cudaFree(p->d_ids);
@@ -178,6 +182,7 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
   std::vector<WarpDesc> warps;
   std::vector<uint32_t> lists;
   std::vector<uint64_t> rec_nblk;
+  std::vector<uint32_t> rec_mul;
   for (ChunkDesc& d : chunks) {
     d.blk_begin = 0;
     d.first_rec = 0;
@@ -234,6 +239,7 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
             if (d.n_recs == 0) d.first_rec = static_cast<uint32_t>(rec_nblk.size());
             d.n_recs += 1;
             rec_nblk.push_back(n);
+            rec_mul.push_back(host_xpow8(d.len - (bb - d.blk_begin + n) * kBlockBytes));
             bb += n;
             if (bb == end) ++j;
           }
@@ -249,6 +255,7 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
   if (e == cudaSuccess) e = upload(&D.d_warps, warps);
   if (e == cudaSuccess) e = upload(&D.d_lists, lists);
   if (e == cudaSuccess) e = upload(&D.d_rec_nblk, rec_nblk);
+  if (e == cudaSuccess) e = upload(&D.d_rec_mul, rec_mul);
   const uint64_t slots = std::max<uint64_t>(D.n_recs, min_recs);
   if (e == cudaSuccess && slots) e = cudaMalloc(&D.d_recs, slots * sizeof(Record));
   return e;
@@ -284,6 +291,8 @@ fr_status run_batches(fr_plan p, const Decomp& D, int mode, uint8_t* packed, FpE
   fp.recs = D.d_recs;
   fp.segs = p->d_segs;
   fp.rec_nblk = D.d_rec_nblk;
+  fp.rec_mul = D.d_rec_mul;
+  fp.crc_xor = p->d_crc_xor;
   fp.n_chunks = p->n_chunks;
   fp.c_begin = D.batches[b0].c_begin;
   fp.c_end = D.batches[b1 - 1].c_end;
@@ -316,6 +325,8 @@ fr_status run_list(fr_plan p, int mode, const uint32_t* ids, uint64_t n, uint8_t
   fp.recs = p->whole.d_recs;
   fp.segs = p->d_segs;
   fp.rec_nblk = nullptr;
+  fp.rec_mul = nullptr;
+  fp.crc_xor = p->d_crc_xor;
   fp.n_chunks = p->n_chunks;
   fp.c_begin = 0;
   fp.c_end = n;
@@ -498,6 +509,11 @@ fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, u
     }
   }
   if (e == cudaSuccess && p->n_segs) e = cudaMalloc(&p->d_segs, p->n_segs * sizeof(double));
+  if (e == cudaSuccess && n_chunks) {
+    std::vector<uint32_t> crc_xor(n_chunks);
+    for (uint64_t c = 0; c < n_chunks; ++c) crc_xor[c] = host_crc_xor_term(p->chunks[c].len);
+    e = upload(&p->d_crc_xor, crc_xor);
+  }
   if (e == cudaSuccess && n_chunks) e = cudaMalloc(&p->d_flags, n_chunks);
   if (e == cudaSuccess && n_chunks) e = cudaMalloc(&p->d_ids, n_chunks * sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMalloc(&p->d_count, sizeof(uint64_t));

@@ -37,6 +37,7 @@ constexpr unsigned kFull = 0xFFFFFFFFu;
 
 __device__ const ByteTable g_byte = make_byte_table();
 __device__ const PowTables g_pow = make_pow_tables();
+__device__ const TailMuls g_tail = make_tail_muls();
 
 // a * b mod P, both variable.
 __device__ __forceinline__ uint32_t gmul(uint32_t a, uint32_t b) {
@@ -67,21 +68,39 @@ __device__ __forceinline__ uint32_t crc_byte(const uint32_t* T, uint32_t r, uint
   return T[(r ^ b) & 0xFFu] ^ (r >> 8);
 }
 
-__device__ __forceinline__ void exact_elem(uint32_t dtype, uint32_t bits, uint32_t& nf, double& s) {
+// (hi, lo) += (bh, bl) as unevaluated float pairs: TwoSum of the high parts,
+// the low parts and the rounding error added in fp32.
+__device__ __forceinline__ void two_sum_pair(float& hi, float& lo, float bh, float bl) {
+  const float t = hi + bh;
+  const float z = t - hi;
+  const float err = (hi - (t - z)) + (bh - z);
+  lo = (lo + bl) + err;
+  hi = t;
+}
+
+// One tail element of type `dtype` with bit pattern `bits`: counted if
+// non-finite, else its square added exactly -- as an fp32 product and its FMA
+// residual into the float pair (hi, lo) when |x| lies in [2^-40, 2^56] (the
+// residual is not subnormal, and 32 lanes of 8 squares stay below 2^120), else
+// in fp64 into dx (rare).  The common case stays off GB300's narrow fp64 pipe.
+__device__ __forceinline__ void tail_elem(uint32_t dtype, uint32_t bits, uint32_t& nf, float& hi, float& lo,
+                                          double& dx) {
+  uint32_t f;
   if (dtype == kDtF32) {
-    if ((bits & 0x7F800000u) == 0x7F800000u) {
-      ++nf;
-    } else {
-      const double x = static_cast<double>(__uint_as_float(bits));
-      s = __dadd_rn(s, __dmul_rn(x, x));
-    }
+    if ((bits & 0x7F800000u) == 0x7F800000u) { ++nf; return; }
+    f = bits;
   } else {
-    if ((bits & 0x7F80u) == 0x7F80u) {
-      ++nf;
-    } else {
-      const double x = static_cast<double>(__uint_as_float(bits << 16));
-      s = __dadd_rn(s, __dmul_rn(x, x));
-    }
+    if ((bits & 0x7F80u) == 0x7F80u) { ++nf; return; }
+    f = bits << 16;
+  }
+  const float x = __uint_as_float(f);
+  const float ax = fabsf(x);
+  if (ax >= 0x1p-40f && ax <= 0x1p56f) {
+    const float p2 = x * x;
+    two_sum_pair(hi, lo, p2, __fmaf_rn(x, x, -p2));
+  } else if (ax != 0.0f) {
+    const double d = static_cast<double>(x);
+    dx = __dadd_rn(dx, __dmul_rn(d, d));
   }
 }
 
@@ -103,12 +122,25 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
     const uint64_t first_rec = p.ids ? pos : cd.first_rec;
     const int64_t n_recs = p.ids ? (body ? 1 : 0) : cd.n_recs;
 
-    // ---- 1. records, last batch first so the byte count after each is known
+    // ---- 1. records: each shifted by the bytes after it in the chunk -- a
+    // multiplier the plan precomputed, or (list mode, no-allocation entry)
+    // found here, last batch of 32 first so the byte count after each is known
     uint32_t raw = 0;
     double sq_rec = 0.0;
     uint32_t nf_rec = 0;
     uint64_t carry = tail;
-    for (int64_t hi = n_recs; hi > 0;) {
+    if (p.rec_mul && !p.ids) {
+      uint32_t n = 0;
+      for (int64_t i = lane; i < n_recs; i += 32) {
+        const Record rec = p.recs[first_rec + i];
+        raw ^= gmul(rec.crc, p.rec_mul[first_rec + i]);
+        n += rec.nonfinite;
+      }
+#pragma unroll
+      for (int m = 16; m >= 1; m >>= 1) n += __shfl_down_sync(kFull, n, m);
+      nf_rec = __shfl_sync(kFull, n, 0);
+    }
+    for (int64_t hi = (p.rec_mul && !p.ids) ? 0 : n_recs; hi > 0;) {
       const int64_t lo = hi > 32 ? hi - 32 : 0;
       const int64_t i = lo + lane;
       const bool have = i < hi;
@@ -134,12 +166,30 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
     }
     // the body's segment sums, in an order fixed by segment index alone
     if (values) {
+      // pair-form slots are added as float pairs (TwoSum), tagged fp64 slots
+      // (rare) in fp64, so the common case stays off the narrow fp64 pipe
       const uint64_t n_seg = (body / kBlockBytes + kSegBlocks - 1) / kSegBlocks;
-      double s = 0.0;
-      for (uint64_t k = lane; k < n_seg; k += 32) s += seg_value(p.segs + cd.seg_base + k);
+      float hi = 0.0f, lo = 0.0f;
+      double dx = 0.0;
+      for (uint64_t k = lane; k < n_seg; k += 32) {
+        const double* slot = p.segs + cd.seg_base + k;
+        if (*reinterpret_cast<const uint64_t*>(slot) >> 63) {
+          dx += seg_value(slot);
+        } else {
+          const float2 f = *reinterpret_cast<const float2*>(slot);  // (lo, hi)
+          two_sum_pair(hi, lo, f.y, f.x);
+        }
+      }
 #pragma unroll
-      for (int m = 16; m >= 1; m >>= 1) s += __shfl_down_sync(kFull, s, m);
-      sq_rec = s;
+      for (int m = 16; m >= 1; m >>= 1) {
+        const float oh = __shfl_down_sync(kFull, hi, m), ol = __shfl_down_sync(kFull, lo, m);
+        two_sum_pair(hi, lo, oh, ol);
+      }
+      if (__any_sync(kFull, dx != 0.0)) {
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) dx += __shfl_down_sync(kFull, dx, m);
+      }
+      sq_rec = (static_cast<double>(hi) + static_cast<double>(lo)) + dx;
     }
 
     // ---- 2. tail
@@ -152,11 +202,16 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
       tsrc = reinterpret_cast<const uint8_t*>(cd.addr) + body;
       if (MODE == kModePack) tdst = p.packed + cd.payload_off + body;
     }
-    double sq_tail = 0.0;
+    // lane l takes the 16-byte piece that ends 16 * (31 - l) bytes before the
+    // tail's end (bytes before the tail are skipped: zero bytes leave a raw
+    // CRC run from zero unchanged), so its shift is a constant
+    float th = 0.0f, tl = 0.0f;  // the tail's sum of squares, as a float pair
+    double tdx = 0.0;            // and its rare fp64 part
     uint32_t nf_tail = 0;
-    const uint32_t b0 = lane * 16u;
-    if (b0 < tail) {
-      const uint32_t b1 = (b0 + 16u < tail) ? b0 + 16u : tail;
+    const int32_t e1 = static_cast<int32_t>(tail) - 16 * (31 - static_cast<int32_t>(lane));
+    if (e1 > 0) {
+      const uint32_t b1 = static_cast<uint32_t>(e1);
+      const uint32_t b0 = b1 > 16u ? b1 - 16u : 0u;
       uint32_t r = 0, word = 0;
       for (uint32_t j = b0; j < b1; ++j) {
         const uint32_t v = __ldg(tsrc + j);
@@ -165,25 +220,31 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
         word |= v << (8 * (j & 3u));
         if (values) {
           if (cd.dtype == kDtF32 && (j & 3u) == 3u) {
-            exact_elem(kDtF32, word, nf_tail, sq_tail);
+            tail_elem(kDtF32, word, nf_tail, th, tl, tdx);
             word = 0;
           } else if (cd.dtype == kDtBf16 && (j & 1u) == 1u) {
-            exact_elem(kDtBf16, word >> (8 * ((j - 1) & 3u)), nf_tail, sq_tail);
+            tail_elem(kDtBf16, (word >> (8 * ((j - 1) & 3u))) & 0xFFFFu, nf_tail, th, tl, tdx);
             if ((j & 3u) == 3u) word = 0;
           }
         }
       }
-      raw ^= shift_bytes(r, tail - b1);
+      raw ^= gmul(r, g_tail.m[lane]);
     }
 #pragma unroll
     for (int m = 16; m >= 1; m >>= 1) {
       raw ^= __shfl_xor_sync(kFull, raw, m);
-      sq_tail += __shfl_down_sync(kFull, sq_tail, m);
       nf_tail += __shfl_down_sync(kFull, nf_tail, m);
+      const float oh = __shfl_down_sync(kFull, th, m), ol = __shfl_down_sync(kFull, tl, m);
+      two_sum_pair(th, tl, oh, ol);
     }
+    if (__any_sync(kFull, tdx != 0.0)) {
+#pragma unroll
+      for (int m = 16; m >= 1; m >>= 1) tdx += __shfl_down_sync(kFull, tdx, m);
+    }
+    const double sq_tail = (static_cast<double>(th) + static_cast<double>(tl)) + tdx;
 
     // ---- 3. preset and final XOR
-    const uint32_t crc = raw ^ shift_bytes(0xFFFFFFFFu, cd.len) ^ 0xFFFFFFFFu;
+    const uint32_t crc = raw ^ (p.crc_xor ? p.crc_xor[c] : (shift_bytes(0xFFFFFFFFu, cd.len) ^ 0xFFFFFFFFu));
     const double sumsq = sq_rec + sq_tail;  // lane 0 holds the fixed-order sums
     const uint32_t nonfinite = nf_rec + nf_tail;
 
@@ -273,9 +334,18 @@ constexpr int kCompactThreads = 1024;
 constexpr int kPerThread = 8;
 constexpr int kTile = kCompactThreads * kPerThread;
 
+// Bulk prefetch of [p, p + bytes) into L2 (bytes rounded down to 16).
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint64_t bytes) {
+  const uint32_t b = static_cast<uint32_t>(bytes) & ~15u;
+  if (b) asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(b) : "memory");
+}
+
 struct FlagPred {
   const uint8_t* flags;
   __device__ __forceinline__ bool operator()(uint64_t i) const { return flags[i] != 0; }
+  __device__ __forceinline__ void prefetch(uint64_t first, uint64_t count) const {
+    prefetch_l2_bulk(flags + first, count);
+  }
 };
 
 struct DiffPred {
@@ -285,11 +355,17 @@ struct DiffPred {
     const uint4 x = a[i], y = b[i];
     return ((x.x ^ y.x) | (x.y ^ y.y) | (x.z ^ y.z) | (x.w ^ y.w)) != 0u;
   }
+  __device__ __forceinline__ void prefetch(uint64_t first, uint64_t count) const {
+    prefetch_l2_bulk(a + first, count * 16);
+    prefetch_l2_bulk(b + first, count * 16);
+  }
 };
 
-// One CTA walks the index space in tiles of kTile; thread t tests kPerThread
-// consecutive indices of the tile, a block-wide exclusive scan of the per-thread
-// counts gives each thread its output position, and the ids are written in
+// One CTA walks the index space in tiles of kTile.  Warp w tests the 256
+// indices [tile + 256w, tile + 256w + 256) in kPerThread rounds, lane l taking
+// index 32j + l in round j, so every load of a round is coalesced; the ballots
+// of the rounds give each hit its rank inside the warp, a block-wide scan of
+// the warp totals gives the warp's output position, and the ids are written in
 // ascending order.  Deterministic: no atomics decide any position.
 template <class Pred>
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(Pred pred, uint64_t n, uint32_t* out,
@@ -298,21 +374,26 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(Pred pred, uin
   __shared__ uint32_t warp_tot[kCompactThreads / 32];
   __shared__ uint64_t base_sh;
   const uint32_t tid = threadIdx.x, lane = tid & 31u, warp = tid >> 5;
+  const uint32_t lt = (1u << lane) - 1u;  // lanes below this one
   uint64_t base = 0;
+  if (tid == 0) pred.prefetch(0, n < kTile ? n : kTile);
   for (uint64_t t0 = 0; t0 < n; t0 += kTile) {
-    const uint64_t first = t0 + static_cast<uint64_t>(tid) * kPerThread;
-    uint32_t bits = 0;
+    // the next tile streams into L2 while this one is tested
+    if (tid == 0 && t0 + kTile < n) pred.prefetch(t0 + kTile, n - (t0 + kTile) < kTile ? n - (t0 + kTile) : kTile);
+    const uint64_t wbase = t0 + static_cast<uint64_t>(warp) * (32 * kPerThread);
+    uint32_t mask[kPerThread];
+    uint32_t total = 0;
+    // branch-free, so all rounds' loads can be in flight at once (indices
+    // past the end test entry 0 and are masked off)
 #pragma unroll
-    for (int j = 0; j < kPerThread; ++j)
-      if (first + j < n && pred(first + j)) bits |= 1u << j;
-    const uint32_t cnt = __popc(bits);
-    uint32_t inc = cnt;
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-      const uint32_t v = __shfl_up_sync(kFull, inc, d);
-      if (lane >= static_cast<uint32_t>(d)) inc += v;
+    for (int j = 0; j < kPerThread; ++j) {
+      const uint64_t i = wbase + 32u * j + lane;
+      const bool in = i < n;
+      const bool hit = pred(in ? i : 0);
+      mask[j] = __ballot_sync(kFull, in && hit);
+      total += __popc(mask[j]);
     }
-    if (lane == 31) warp_tot[warp] = inc;
+    if (lane == 0) warp_tot[warp] = total;
     __syncthreads();
     if (warp == 0) {
       uint32_t w = warp_tot[lane];
@@ -326,12 +407,14 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(Pred pred, uin
       if (lane == 31) base_sh = base + winc;
     }
     __syncthreads();
-    uint64_t pos = base + warp_tot[warp] + (inc - cnt);
-    while (bits) {
-      const int j = __ffs(bits) - 1;
-      bits &= bits - 1;
-      if (pos < cap) out[pos] = static_cast<uint32_t>(first + j);
-      ++pos;
+    uint64_t pos = base + warp_tot[warp];
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      if ((mask[j] >> lane) & 1u) {
+        const uint64_t q = pos + __popc(mask[j] & lt);
+        if (q < cap) out[q] = static_cast<uint32_t>(wbase + 32u * j + lane);
+      }
+      pos += __popc(mask[j]);
     }
     base = base_sh;
     __syncthreads();

@@ -240,6 +240,8 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
   fp.recs = d_recs;
   fp.segs = reinterpret_cast<const double*>(scratch + kOffSegs);
   fp.rec_nblk = reinterpret_cast<const uint64_t*>(scratch + kOffRecNblk);
+  fp.rec_mul = nullptr;  // shifts and CRC terms are computed in the finalize kernel
+  fp.crc_xor = nullptr;
   fp.n_chunks = n_chunks;
   fp.c_begin = 0;
   fp.c_end = n_chunks;

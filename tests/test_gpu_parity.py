@@ -126,6 +126,16 @@ def test_special_values():
     spiky[12345] = 1e-20
     cases.append(spiky)
     got, want = compare_full(cases, 16 * KiB)
+    # the same values in tensors with a 148-byte (fp32) / 74-byte (bf16) tail,
+    # on both sides of the tail's fp32 range [2^-40, 2^56]
+    tails = [torch.full((4096 + 37,), v, device="cuda") for v in
+             (1e-12, 8e-13, 3e16, 1e17, 3e19, 1e-25, 1e-40, float("nan"), 0.5)]
+    tails += [torch.full((8192 + 37,), v, device="cuda").to(torch.bfloat16) for v in (1e-12, 3e16, 1e17, 3e19)]
+    mixed_t = torch.randn(4096 + 37, device="cuda")
+    mixed_t[-37::5] = 2e30
+    mixed_t[-36::7] = float("inf")
+    tails.append(mixed_t)
+    compare_full(tails, 16 * KiB)
     t = table_np(got["table"])
     per = (n * 4) // (16 * KiB)
     assert (t["sumsq"][:per] == 0).all()
