@@ -48,7 +48,7 @@ struct BatchInfo {
 // decomposition's block offsets and record ranges.
 struct Decomp {
   int n_ctas = 0;
-  uint32_t n_warps = 0;  // per class launch: n_ctas * kSweepWarps
+  uint32_t n_warps = 0;  // per class launch: n_ctas * warps per CTA
   std::vector<BatchInfo> batches;
   uint64_t n_recs = 0;
   ChunkDesc* d_chunks = nullptr;
@@ -67,8 +67,12 @@ struct fr_plan_s {
   uint64_t chunk_bytes = 0, n_chunks = 0, packed_bytes = 0, state_bytes = 0;
   uint32_t n_batches = 1;
   std::vector<ChunkDesc> chunks;  // layout fields (host copy)
-  Decomp whole;                   // one batch over all SMs
-  Decomp batched;                 // n_batches > 1: batches over half the SMs
+  // Decompositions, one per distinct warps-per-CTA count of the sweep modes
+  // (geo[mode] indexes them): whole = one batch over all SMs; batched (when
+  // n_batches > 1) = batches over half the SMs.  whole[0] also holds n_chunks
+  // record slots for list-mode calls.
+  std::vector<Decomp> whole, batched;
+  int geo[4] = {0, 0, 0, 0};
   uint64_t n_segs = 0;            // 16 KiB sum segments of all chunk bodies
   double* d_segs = nullptr;       // their sums of squares
   uint32_t* d_crc_xor = nullptr;  // per chunk: the CRC preset/final-XOR term of its length
@@ -155,8 +159,8 @@ void free_decomp(Decomp& D) {
 }
 
 void free_device(fr_plan p) {
-  free_decomp(p->whole);
-  free_decomp(p->batched);
+  for (Decomp& d : p->whole) free_decomp(d);
+  for (Decomp& d : p->batched) free_decomp(d);
   cudaFree(p->d_segs);
   cudaFree(p->d_crc_xor);
   cudaFree(p->d_flags);
@@ -174,8 +178,9 @@ void free_device(fr_plan p) {
 // by class, so each chunk's records are consecutive.  `min_recs`: record slots
 // to allocate at least (list-mode calls use one slot per listed chunk).
 cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<uint64_t>& bounds, int n_ctas,
+                         int warps_per_cta,
                          uint64_t min_recs, Decomp& D) {
-  const uint64_t W = static_cast<uint64_t>(n_ctas) * kSweepWarps;
+  const uint64_t W = static_cast<uint64_t>(n_ctas) * warps_per_cta;
   D.n_ctas = n_ctas;
   D.n_warps = static_cast<uint32_t>(W);
   std::vector<ChunkDesc> chunks = base;
@@ -312,17 +317,17 @@ fr_status run_list(fr_plan p, int mode, const uint32_t* ids, uint64_t n, uint8_t
                    cudaStream_t s) {
   if (n == 0) return FR_OK;
   ListParams lp;
-  lp.chunks = p->whole.d_chunks;
+  lp.chunks = p->whole[0].d_chunks;
   lp.ids = ids;
   lp.n = n;
-  lp.recs = p->whole.d_recs;
+  lp.recs = p->whole[0].d_recs;
   lp.segs = p->d_segs;
   lp.packed = packed;
   cudaError_t e = launch_list_sweep(mode, lp, s);
   if (e != cudaSuccess) return cuda_fail(e, "list sweep kernel launch");
   FinalizeParams fp;
-  fp.chunks = p->whole.d_chunks;
-  fp.recs = p->whole.d_recs;
+  fp.chunks = p->whole[0].d_chunks;
+  fp.recs = p->whole[0].d_recs;
   fp.segs = p->d_segs;
   fp.rec_nblk = nullptr;
   fp.rec_mul = nullptr;
@@ -353,7 +358,11 @@ fr_status check_packed_buffer(fr_plan p, const void* buf, uint64_t bytes) {
   return FR_OK;
 }
 
-const Decomp& batch_decomp(fr_plan p) { return p->n_batches > 1 ? p->batched : p->whole; }
+// The decomposition a mode's whole-state / batch calls run on.
+const Decomp& whole_for(fr_plan p, int mode) { return p->whole[p->geo[mode]]; }
+const Decomp& batch_for(fr_plan p, int mode) {
+  return p->n_batches > 1 ? p->batched[p->geo[mode]] : p->whole[p->geo[mode]];
+}
 
 fr_status check_same_layout(fr_plan src, fr_plan dst) {
   if (src->device != dst->device || src->n_chunks != dst->n_chunks || src->packed_bytes != dst->packed_bytes ||
@@ -491,7 +500,18 @@ fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, u
   // ---- decompositions
   e = cudaSuccess;
   if (n_chunks > 0) {
-    e = build_decomp(p->chunks, {0, n_chunks}, n_sm, n_chunks, p->whole);
+    std::vector<int> counts;  // distinct warps-per-CTA counts of the modes
+    for (int m = 0; m < 4; ++m) {
+      const int w = sweep_warps(m);
+      int g = 0;
+      while (g < static_cast<int>(counts.size()) && counts[g] != w) ++g;
+      if (g == static_cast<int>(counts.size())) counts.push_back(w);
+      p->geo[m] = g;
+    }
+    p->whole.resize(counts.size());
+    p->batched.resize(counts.size());
+    for (size_t g = 0; e == cudaSuccess && g < counts.size(); ++g)
+      e = build_decomp(p->chunks, {0, n_chunks}, n_sm, counts[g], g == 0 ? n_chunks : 0, p->whole[g]);
     if (e == cudaSuccess && p->n_batches > 1) {
       // batch starts at about equal state bytes, every batch non-empty
       std::vector<uint64_t> bounds(1, 0);
@@ -505,7 +525,8 @@ fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, u
       bounds.push_back(n_chunks);
       for (size_t i = 1; i < bounds.size(); ++i)
         if (bounds[i] <= bounds[i - 1]) bounds[i] = bounds[i - 1] + 1;
-      e = build_decomp(p->chunks, bounds, std::max(1, n_sm / 2), 0, p->batched);
+      for (size_t g = 0; e == cudaSuccess && g < counts.size(); ++g)
+        e = build_decomp(p->chunks, bounds, std::max(1, n_sm / 2), counts[g], 0, p->batched[g]);
     }
   }
   if (e == cudaSuccess && p->n_segs) e = cudaMalloc(&p->d_segs, p->n_segs * sizeof(double));
@@ -566,7 +587,7 @@ fr_status fr_plan_batch(fr_plan p, uint32_t batch, uint32_t* n_batches, uint64_t
     return FR_OK;
   }
   if (batch >= p->n_batches) return invalid("batch out of range");
-  const BatchInfo& b = batch_decomp(p).batches[batch];
+  const BatchInfo& b = batch_for(p, kModePack).batches[batch];
   if (first_chunk) *first_chunk = b.c_begin;
   if (n_chunks) *n_chunks = b.c_end - b.c_begin;
   return FR_OK;
@@ -586,7 +607,7 @@ fr_status fr_fingerprint(fr_plan p, fr_fp* out_dev, void* stream) {
   if (out_dev == nullptr) return invalid("out_dev is null");
   DeviceGuard g(p->device);
   if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
-  return run_batches(p, p->whole, kModeFingerprint, nullptr, reinterpret_cast<FpEntry*>(out_dev), 0, 1,
+  return run_batches(p, whole_for(p, kModeFingerprint), kModeFingerprint, nullptr, reinterpret_cast<FpEntry*>(out_dev), 0, 1,
                      static_cast<cudaStream_t>(stream));
 }
 
@@ -601,7 +622,7 @@ fr_status fr_pack_fp(fr_plan p, void* dst, uint64_t dst_bytes, fr_fp* fp_dev, vo
   if (st != FR_OK) return st;
   DeviceGuard g(p->device);
   if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
-  return run_batches(p, p->whole, kModePack, static_cast<uint8_t*>(dst), reinterpret_cast<FpEntry*>(fp_dev), 0, 1,
+  return run_batches(p, whole_for(p, kModePack), kModePack, static_cast<uint8_t*>(dst), reinterpret_cast<FpEntry*>(fp_dev), 0, 1,
                      static_cast<cudaStream_t>(stream));
 }
 
@@ -624,7 +645,8 @@ fr_status fr_unpack_verify_fp(fr_plan p, const void* src, uint64_t src_bytes, ui
   }
   fr_status st = check_packed_buffer(p, src, src_bytes);
   if (st != FR_OK) return st;
-  st = run_batches(p, p->whole, fp_dev ? kModeUnpackFp : kModeUnpack,
+  const int mode = fp_dev ? kModeUnpackFp : kModeUnpack;
+  st = run_batches(p, whole_for(p, mode), mode,
                    const_cast<uint8_t*>(static_cast<const uint8_t*>(src)), reinterpret_cast<FpEntry*>(fp_dev), 0, 1, s);
   if (st != FR_OK) return st;
   cudaError_t e = launch_compact_flags(p->d_flags, p->n_chunks, mismatch_dev, cap, n_mismatch_dev, p->d_status, s);
@@ -639,7 +661,7 @@ fr_status fr_pack_batch(fr_plan p, uint32_t batch, void* dst, uint64_t dst_bytes
   if (st != FR_OK) return st;
   DeviceGuard g(p->device);
   if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
-  return run_batches(p, batch_decomp(p), kModePack, static_cast<uint8_t*>(dst), nullptr, batch, batch + 1,
+  return run_batches(p, batch_for(p, kModePack), kModePack, static_cast<uint8_t*>(dst), nullptr, batch, batch + 1,
                      static_cast<cudaStream_t>(stream));
 }
 
@@ -651,7 +673,7 @@ fr_status fr_unpack_verify_batch(fr_plan p, uint32_t batch, const void* src, uin
   if (st != FR_OK) return st;
   DeviceGuard g(p->device);
   if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
-  return run_batches(p, batch_decomp(p), kModeUnpack, const_cast<uint8_t*>(static_cast<const uint8_t*>(src)),
+  return run_batches(p, batch_for(p, kModeUnpack), kModeUnpack, const_cast<uint8_t*>(static_cast<const uint8_t*>(src)),
                      nullptr, batch, batch + 1, static_cast<cudaStream_t>(stream));
 }
 
@@ -696,10 +718,10 @@ fr_status fr_restore_fp(fr_plan src, fr_plan dst, void* staging, uint64_t stagin
   st = check_packed_buffer(src, staging, staging_bytes);
   if (st != FR_OK) return st;
   uint8_t* buf = static_cast<uint8_t*>(staging);
-  const Decomp& DS = batch_decomp(src);
-  const Decomp& DD = batch_decomp(dst);
   FpEntry* fs = reinterpret_cast<FpEntry*>(fp_src_dev);
   FpEntry* fd = reinterpret_cast<FpEntry*>(fp_dst_dev);
+  const Decomp& DS = batch_for(src, kModePack);
+  const Decomp& DD = batch_for(dst, fd ? kModeUnpackFp : kModeUnpack);
   cudaError_t e;
   // Pipeline: batch b is unpacked on the receiver's stream as soon as the
   // replica's stream has packed it, while the replica packs batch b+1.

@@ -43,11 +43,28 @@ struct FinalizeParams {
   uint8_t* flags;   // unpack: per-chunk verdict
 };
 
-// Geometry of the sweep kernel: one CTA of kSweepWarps warps per SM.
-#ifndef FR_SWEEP_WARPS
-#define FR_SWEEP_WARPS 16
+// Geometry of the sweep kernels: one CTA per SM, with a warp count per mode
+// (measured on GB300 with the 31.8 GB shard: the issue-bound fingerprint
+// wants 16 warps with deep per-warp stages -- 20 warps cost it 7 points; the
+// latency-bound pack and unpack want 20 warps in flight -- 2 points more).
+#ifndef FR_WARPS_FP
+#define FR_WARPS_FP 16
 #endif
-constexpr int kSweepWarps = FR_SWEEP_WARPS;
+#ifndef FR_WARPS_PACK
+#define FR_WARPS_PACK 20
+#endif
+#ifndef FR_WARPS_UNPACK
+#define FR_WARPS_UNPACK 20
+#endif
+#ifndef FR_WARPS_UNPACK_FP
+#define FR_WARPS_UNPACK_FP 20
+#endif
+__host__ __device__ constexpr int sweep_warps(int mode) {
+  return mode == kModeFingerprint ? FR_WARPS_FP
+         : mode == kModePack      ? FR_WARPS_PACK
+         : mode == kModeUnpack    ? FR_WARPS_UNPACK
+                                  : FR_WARPS_UNPACK_FP;
+}
 
 // Per device, before the first launch: opt the sweep kernels in to their
 // shared-memory size.

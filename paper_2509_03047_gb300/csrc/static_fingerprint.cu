@@ -37,7 +37,7 @@ namespace {
 
 // Limits of the static variant.
 constexpr uint64_t kMaxChunks = FR_STATIC_MAX_CHUNKS;
-constexpr uint64_t kMaxWarpsPerClass = 160 * kSweepWarps;  // up to 160 SMs
+constexpr uint64_t kMaxWarpsPerClass = 160 * sweep_warps(kModeFingerprint);  // up to 160 SMs
 constexpr uint64_t kClasses = 6;
 constexpr uint64_t kMaxWarps = kClasses * kMaxWarpsPerClass;
 constexpr uint64_t kMaxRecs = kMaxWarps + kMaxChunks;
@@ -128,7 +128,7 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
   int n_sm = 0;
   e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
-  const uint64_t W = static_cast<uint64_t>(n_sm) * kSweepWarps;
+  const uint64_t W = static_cast<uint64_t>(n_sm) * sweep_warps(kModeFingerprint);
   if (W > kMaxWarpsPerClass) return fail(FR_ERR_INVALID_ARG, "GPU has more SMs than the static tables hold");
 
   std::lock_guard<std::mutex> lk(g_mu);

@@ -23,8 +23,9 @@
 //    fp64 from a reload of its 16-byte units, so the fast path never needs a
 //    per-element test.
 //
-// No tensor cores: nothing here is a contraction.  One CTA of 16 warps per SM
-// (the 128 KiB of lane-replicated tables fill most of shared memory).  The
+// No tensor cores: nothing here is a contraction.  One CTA per SM, with a warp
+// count per mode (the 128 KiB of lane-replicated tables fill most of shared
+// memory).  The
 // plan sorts chunks into classes by element type and by whether the tensor
 // is 16-byte aligned; each class gets its own block stream, cut into equal
 // per-warp ranges, and its own kernel specialization, so every kernel holds a
@@ -44,22 +45,27 @@ namespace frk {
 
 namespace {
 
-constexpr int kWarps = kSweepWarps;
-constexpr int kThreads = kWarps * 32;
+// Warps and threads of one mode's CTA.
+template <int MODE>
+struct Cta {
+  static constexpr int kWarps = sweep_warps(MODE);
+  static constexpr int kThreads = kWarps * 32;
+};
 constexpr int kTableBytes = 4 * 256 * 32 * 4;  // 4 tables x 256 entries x 32 lanes x 4 B
 // Pipeline geometry (compile-time), tuned on GB300 by timing the 31.8 GB
-// Llama-70B shard.  The read-only fingerprint gains from bulk L2 prefetch one
-// span ahead; pack and unpack lose by it (their write stream evicts the
-// prefetched lines before use, and DRAM reads grow by ~20%), so they rely on
-// register stages alone, unpack with a deeper one.
+// Llama-70B shard.  The read-only fingerprint gains from bulk L2 prefetch
+// exactly one span ahead (none: -9 points; two spans: -25) and from 8-block
+// register stages; pack and unpack lose by the prefetch (their write stream
+// evicts the prefetched lines before use, and DRAM reads grow by ~20%), so
+// they rely on 4-block register stages and more warps (kernels.h).
 #ifndef FR_STAGE_FP
-#define FR_STAGE_FP 4
+#define FR_STAGE_FP 8
 #endif
 #ifndef FR_STAGE_PACK
 #define FR_STAGE_PACK 4
 #endif
 #ifndef FR_STAGE_UNPACK
-#define FR_STAGE_UNPACK 8
+#define FR_STAGE_UNPACK 4
 #endif
 #ifndef FR_AHEAD_FP
 #define FR_AHEAD_FP 1
@@ -96,7 +102,7 @@ extern __shared__ __align__(16) uint8_t g_smem[];
 // i.e. bank l.  The address of (table k, byte k of x, this lane) is one
 // byte-permute: byte 0 = l*4, byte 1 = byte k of x.
 __device__ __forceinline__ void fill_tables() {
-  for (int q = threadIdx.x; q < kTableBytes / 16; q += kThreads) {
+  for (int q = threadIdx.x; q < kTableBytes / 16; q += blockDim.x) {
     const int k = q >> 11, rem = q & 2047, i = rem >> 3, g = rem & 7;
     const uint32_t v = g_braid.t[k][i];
     const uint32_t off = (k >> 1) * 65536 + i * 256 + (k & 1) * 128 + g * 16;
@@ -532,11 +538,11 @@ __device__ __forceinline__ void sweep_piece_al(const uint8_t* tensor, uint8_t* p
 // tensor of the class is 16-byte aligned (128-bit loads and stores); else the
 // tensor side uses 32-bit or byte accesses, chosen per piece.
 template <int MODE, int DT, bool ALIGNED>
-__global__ void __launch_bounds__(kThreads, 1) sweep_kernel(SweepParams p) {
+__global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_kernel(SweepParams p) {
   fill_tables();
   __syncthreads();
   const uint32_t lane = threadIdx.x & 31u;
-  const uint32_t w = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  const uint32_t w = blockIdx.x * Cta<MODE>::kWarps + (threadIdx.x >> 5);
   if (w >= p.n_warps) return;
   const WarpDesc wd = p.warps[w];
   uint64_t b = wd.blk_begin, left = wd.nblk;
@@ -578,11 +584,11 @@ __device__ __noinline__ void list_piece(const uint8_t* tensor, uint8_t* packed, 
 }
 
 template <int MODE>
-__global__ void __launch_bounds__(kThreads, 1) list_kernel(ListParams p) {
+__global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) list_kernel(ListParams p) {
   fill_tables();
   __syncthreads();
   const uint32_t lane = threadIdx.x & 31u;
-  const uint64_t w = static_cast<uint64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+  const uint64_t w = static_cast<uint64_t>(blockIdx.x) * Cta<MODE>::kWarps + (threadIdx.x >> 5);
   if (w >= p.n) return;
   const ChunkDesc cd = p.chunks[p.ids[w]];
   const uint64_t nb = cd.len / kBlockBytes;
@@ -608,8 +614,8 @@ __global__ void __launch_bounds__(kThreads, 1) list_kernel(ListParams p) {
 template <int MODE>
 cudaError_t launch_list(const ListParams& p, cudaStream_t s) {
   if (p.n == 0) return cudaSuccess;
-  const uint64_t ctas = (p.n + kWarps - 1) / kWarps;
-  list_kernel<MODE><<<static_cast<unsigned>(ctas), kThreads, kTableBytes, s>>>(p);
+  const uint64_t ctas = (p.n + Cta<MODE>::kWarps - 1) / Cta<MODE>::kWarps;
+  list_kernel<MODE><<<static_cast<unsigned>(ctas), Cta<MODE>::kThreads, kTableBytes, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -621,7 +627,7 @@ cudaError_t configure_one() {
 
 template <int MODE, int DT, bool ALIGNED>
 cudaError_t launch_one(const SweepParams& p, int n_ctas, cudaStream_t s) {
-  sweep_kernel<MODE, DT, ALIGNED><<<n_ctas, kThreads, kTableBytes, s>>>(p);
+  sweep_kernel<MODE, DT, ALIGNED><<<n_ctas, Cta<MODE>::kThreads, kTableBytes, s>>>(p);
   return cudaGetLastError();
 }
 
