@@ -21,9 +21,15 @@ controller waits for its optimizer step to finish.  If every replica of a
 failed process is lost too, only a checkpoint can help (the paper's first
 limitation, Sec. III-G).
 
+Failures reach the controller two ways (Sec. III-C): a report (the process
+is gone, or a device plugin says so), or a heartbeat that stops -- a rank
+that hangs without exiting is declared failed once it has been silent for
+`heartbeat_timeout` seconds.
+
 This module is host logic only: the Controller, and a simulation that runs
-ranks as separate CPU processes reporting tags through a torch TCPStore, with
-faults made on the host (a rank exits).  No GPU is involved.
+ranks as separate CPU processes reporting tags and heartbeats through a
+torch TCPStore, with faults made on the host (a rank exits, or hangs without
+exiting).  No GPU is involved.
 """
 from __future__ import annotations
 
@@ -53,8 +59,11 @@ class Controller:
 
     `dp_groups`: lists of ranks that hold replicas of the same model state."""
 
-    def __init__(self, world_size: int, dp_groups: Sequence[Sequence[int]]):
+    def __init__(self, world_size: int, dp_groups: Sequence[Sequence[int]],
+                 heartbeat_timeout: Optional[float] = None):
         self.world_size = world_size
+        self.heartbeat_timeout = heartbeat_timeout
+        self.beats: Dict[int, tuple] = {}  # rank -> (heartbeat count, time it last changed)
         self.group_of: Dict[int, List[int]] = {}
         for g in dp_groups:
             for r in g:
@@ -69,6 +78,26 @@ class Controller:
 
     def report_failure(self, rank: int) -> None:
         self.failed.add(rank)
+
+    def beat(self, rank: int, count: int, now: float) -> None:
+        """A rank's heartbeat counter as last read; only a change counts as a
+        beat, and a rank's clock starts with its first beat (a process still
+        starting up is not silent)."""
+        if count == 0:
+            return
+        old = self.beats.get(rank)
+        if old is None or old[0] != count:
+            self.beats[rank] = (count, now)
+
+    def check_timeouts(self, now: float) -> List[int]:
+        """Declare failed every rank silent for longer than the timeout; returns them."""
+        if self.heartbeat_timeout is None:
+            return []
+        out = [r for r, (_, t) in self.beats.items()
+               if r not in self.failed and now - t > self.heartbeat_timeout]
+        for r in out:
+            self.report_failure(r)
+        return out
 
     def decide(self) -> Optional[Decision]:
         """A decision once it is safe to stop the normal ranks, else None."""
@@ -96,9 +125,11 @@ class Controller:
 # ---------------------------------------------------------------- simulation
 
 def _rank_main(rank: int, world: int, host: str, port: int, n_steps: int, fail_step: int, fail_phase: str,
-               step_time: float) -> None:
+               step_time: float, fail_mode: str = "exit") -> None:
     """One simulated training process.  Its 'model state' is the number of
-    optimizer updates it applied, reported with every tag."""
+    optimizer updates it applied, reported with every tag; it beats its
+    heartbeat counter with every tag and while it waits.  fail_mode "exit":
+    the process dies; "hang": it stays alive but goes silent until stopped."""
     from datetime import timedelta
 
     import torch.distributed as dist
@@ -106,38 +137,52 @@ def _rank_main(rank: int, world: int, host: str, port: int, n_steps: int, fail_s
     store = dist.TCPStore(host, port, world + 1, False, timeout=timedelta(seconds=60))
     updates = 0
 
+    def beat():
+        store.add("hb/%d" % rank, 1)
+
     def tag(t):
         store.set("state/%d" % rank, str(updates))
         store.set("tag/%d" % rank, str(t))
+        beat()
 
     def stopped():
         return store.check(["stop"])
 
+    def fail():
+        if fail_mode == "exit":
+            os._exit(3)  # the fault: this process dies
+        while not stopped():  # the fault: alive, silent
+            time.sleep(0.005)
+
     for i in range(n_steps):
         tag(i)
         if fail_phase == "forward_backward" and i == fail_step:
-            os._exit(3)  # the fault: this process dies
+            return fail()
         time.sleep(step_time)  # forward and backward
         # barrier merged with the gradient all-reduce
         store.add("barrier/%d" % i, 1)
         while int(store.add("barrier/%d" % i, 0)) < world:
             if stopped():
                 return
+            beat()
             time.sleep(0.005)
         tag(OPTIMIZER)
         if fail_phase == "optimizer" and i == fail_step:
-            os._exit(3)
+            return fail()
         time.sleep(step_time / 2)  # the optimizer step
         updates += 1
         tag(i + 1)
     while not stopped():
+        beat()
         time.sleep(0.005)
 
 
 def simulate(world: int, dp_groups: Sequence[Sequence[int]], n_steps: int, fail_rank: int, fail_step: int,
-             fail_phase: str, step_time: float = 0.02, timeout: float = 60.0):
-    """Run `world` CPU ranks; rank `fail_rank` dies in `fail_phase` of step
-    `fail_step`.  Returns (decision, {rank: updates held when stopped})."""
+             fail_phase: str, step_time: float = 0.02, timeout: float = 60.0, fail_mode: str = "exit",
+             heartbeat_timeout: float = 1.0):
+    """Run `world` CPU ranks; rank `fail_rank` dies ("exit") or goes silent
+    ("hang") in `fail_phase` of step `fail_step`.  Returns (decision, {rank:
+    updates held when stopped})."""
     import multiprocessing as mp
     import socket
     from datetime import timedelta
@@ -154,21 +199,25 @@ def simulate(world: int, dp_groups: Sequence[Sequence[int]], n_steps: int, fail_
     procs = []
     for r in range(world):
         fs, fp = (fail_step, fail_phase) if r == fail_rank else (-1, "")
-        procs.append(ctx.Process(target=_rank_main, args=(r, world, "127.0.0.1", port, n_steps, fs, fp, step_time)))
+        procs.append(ctx.Process(target=_rank_main,
+                                 args=(r, world, "127.0.0.1", port, n_steps, fs, fp, step_time, fail_mode)))
     for p in procs:
         p.start()
-    ctl = Controller(world, dp_groups)
+    ctl = Controller(world, dp_groups, heartbeat_timeout=heartbeat_timeout)
     decision = None
     t0 = time.time()
     try:
         while decision is None:
             if time.time() - t0 > timeout:
                 raise TimeoutError("no decision")
+            now = time.time()
             for r, p in enumerate(procs):
                 if p.exitcode not in (None, 0):
                     ctl.report_failure(r)  # the monitoring side: the process is gone
                 if store.check(["tag/%d" % r]):
                     ctl.heartbeat(r, int(store.get("tag/%d" % r)))
+                ctl.beat(r, int(store.add("hb/%d" % r, 0)), now)
+            ctl.check_timeouts(now)  # silent ranks
             decision = ctl.decide()
             time.sleep(0.01)
         store.set("stop", "1")

@@ -61,3 +61,28 @@ def test_simulated_failure_resumes_at_the_right_step(phase, fail_step, resume):
     # every normal replica holds exactly the state of the resume step, so the
     # failed rank restored from its replica agrees with everyone
     assert set(held.values()) == {resume}
+
+
+def test_heartbeat_timeout_declares_a_silent_rank_failed():
+    c = st.Controller(4, GROUPS, heartbeat_timeout=1.0)
+    for r in range(4):
+        c.beat(r, 1, now=0.0)
+        c.heartbeat(r, 7)
+    for r in (0, 2, 3):
+        c.beat(r, 5, now=0.8)  # ranks 0, 2, 3 keep beating; rank 1 falls silent
+        c.beat(r, 5, now=0.9)  # an unchanged counter is not a beat
+    assert c.check_timeouts(now=0.95) == []
+    assert c.check_timeouts(now=1.05) == [1]
+    d = c.decide()
+    assert d.restore == [1] and d.resume_step == 7 and d.source == {1: 3}
+    assert c.check_timeouts(now=1.75) == []
+    assert c.check_timeouts(now=1.85) == [0, 2, 3]  # silent since 0.8
+
+
+@pytest.mark.parametrize("phase,resume", [("forward_backward", 2), ("optimizer", 3)])
+def test_simulated_hang_is_found_by_its_silent_heartbeat(phase, resume):
+    decision, held = st.simulate(world=4, dp_groups=GROUPS, n_steps=6, fail_rank=2, fail_step=2, fail_phase=phase,
+                                 fail_mode="hang", heartbeat_timeout=0.5)
+    assert decision.restore == [2] and decision.source == {2: 0}
+    assert decision.resume_step == resume and decision.phase == phase
+    assert set(held.values()) == {resume}
