@@ -123,16 +123,32 @@ __device__ __forceinline__ uint32_t braid_step(uint32_t x, uint32_t lb) {
   return (t0 ^ t1) ^ (t2 ^ t3);
 }
 
-// a * K mod P for a compile-time K: XOR of K * x^k over the set bits of a.
-template <uint32_t K>
-__device__ __forceinline__ uint32_t mulk(uint32_t a) {
-  uint32_t r = 0, b = K;
-#pragma unroll
-  for (int k = 0; k < 32; ++k) {
-    r ^= b & static_cast<uint32_t>(static_cast<int32_t>(a << k) >> 31);
-    b = gf_mul_x(b);
-  }
-  return r;
+// The piece-end fold multiplies by seven constants: x^32 (Horner inside the
+// lane), x^128 ... x^2048 (the shuffle tree) and the unbraid factor.  Each
+// multiply is four byte lookups in that constant's tables (read-only, cached
+// in L1) instead of a 32-step bit loop: a warp pays the fold once per piece,
+// which matters for states of many small tensors.
+struct FoldTables {
+  ByteTables4 m[7];
+};
+__host__ __device__ constexpr FoldTables make_fold_tables() {
+  FoldTables f{};
+  f.m[0] = make_mul_tables(gf_xpow(32));
+  f.m[1] = make_mul_tables(gf_xpow(128));
+  f.m[2] = make_mul_tables(gf_xpow(256));
+  f.m[3] = make_mul_tables(gf_xpow(512));
+  f.m[4] = make_mul_tables(gf_xpow(1024));
+  f.m[5] = make_mul_tables(gf_xpow(2048));
+  f.m[6] = make_mul_tables(kUnbraid);
+  return f;
+}
+__device__ const FoldTables g_fold = make_fold_tables();
+
+// a * (constant i) mod P.
+__device__ __forceinline__ uint32_t mul_fold(int i, uint32_t a) {
+  const ByteTables4& T = g_fold.m[i];
+  return (__ldg(&T.t[0][a & 255u]) ^ __ldg(&T.t[1][(a >> 8) & 255u])) ^
+         (__ldg(&T.t[2][(a >> 16) & 255u]) ^ __ldg(&T.t[3][a >> 24]));
 }
 
 // ------------------------------------------------------------------ memory
@@ -494,21 +510,21 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
   }
 
   // ---- fold the 128 streams into the raw CRC of the piece
-  uint32_t v = mulk<gf_xpow(32)>(L.s[0]) ^ L.s[1];
-  v = mulk<gf_xpow(32)>(v) ^ L.s[2];
-  v = mulk<gf_xpow(32)>(v) ^ L.s[3];
+  uint32_t v = mul_fold(0, L.s[0]) ^ L.s[1];
+  v = mul_fold(0, v) ^ L.s[2];
+  v = mul_fold(0, v) ^ L.s[3];
   {
     uint32_t o;
     o = __shfl_down_sync(0xFFFFFFFFu, v, 1);
-    v = mulk<gf_xpow(128)>(v) ^ o;
+    v = mul_fold(1, v) ^ o;
     o = __shfl_down_sync(0xFFFFFFFFu, v, 2);
-    v = mulk<gf_xpow(256)>(v) ^ o;
+    v = mul_fold(2, v) ^ o;
     o = __shfl_down_sync(0xFFFFFFFFu, v, 4);
-    v = mulk<gf_xpow(512)>(v) ^ o;
+    v = mul_fold(3, v) ^ o;
     o = __shfl_down_sync(0xFFFFFFFFu, v, 8);
-    v = mulk<gf_xpow(1024)>(v) ^ o;
+    v = mul_fold(4, v) ^ o;
     o = __shfl_down_sync(0xFFFFFFFFu, v, 16);
-    v = mulk<gf_xpow(2048)>(v) ^ o;
+    v = mul_fold(5, v) ^ o;
   }
 
   uint32_t nonfinite = L.nonfinite;
@@ -518,7 +534,7 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
   }
   if (lane == 0) {
     Record r;
-    r.crc = mulk<kUnbraid>(v);
+    r.crc = mul_fold(6, v);
     r.nonfinite = nonfinite;
     r.unused = 0.0;
     *rec = r;
