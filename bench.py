@@ -407,6 +407,26 @@ def run_flashrec(args):
             step(buf=host_buf, sync_counts=True)
         torch.cuda.synchronize()
         t_serial = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
+        # (d) the bound: the host link's copy engines moving P/2 bytes each way
+        # at once (64 MiB pieces, two streams, disjoint halves of the buffers)
+        half, piece = P // 2, 64 << 20
+
+        def link_step():
+            for o in range(0, half, piece):
+                n = min(piece, half - o)
+                with torch.cuda.stream(s_src):
+                    host_buf[o:o + n].copy_(packed[o:o + n], non_blocking=True)
+                with torch.cuda.stream(s_dst):
+                    packed[half + o:half + o + n].copy_(host_buf[half + o:half + o + n], non_blocking=True)
+            torch.cuda.synchronize()
+
+        link_step()
+        t0 = time.perf_counter()
+        for _ in range(2):
+            link_step()
+        t_link = (time.perf_counter() - t0) / 2
+        link_gbs = half / t_link / 1e9
+        restore_gbs = P / t_e2e / 1e9
         e2e = {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_e2e / 1e9, dev), 2), "unit": "GB/s",
                "h2d_bytes_per_step": P, "d2h_bytes_per_step": P + 16, "ms_per_step": round(t_e2e * 1e3, 2),
                "transfer": "pinned host buffer over NVLink-C2C; fr_restore_fp with %d batches, pack and unpack "
@@ -416,6 +436,10 @@ def run_flashrec(args):
                            "ms_per_step": round(t_unfused * 1e3, 2),
                            "how": "fr_fingerprint, fr_restore, fr_fingerprint, fr_diff"},
                "found": {"mismatching_chunks": e2e_found[0], "diverged_chunks": e2e_found[1]},
+               "link": {"copy_engines_each_way_gbs": round(link_gbs, 1),
+                        "restore_each_way_gbs": round(restore_gbs, 1), "frac": round(restore_gbs / link_gbs, 4),
+                        "how": "cudaMemcpyAsync of P/2 bytes device->host and P/2 host->device at once, 64 MiB "
+                               "pieces on two streams, pinned host memory; the restore moves P each way"},
                "serial": {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_serial / 1e9, dev), 2),
                           "ms_per_step": round(t_serial * 1e3, 2),
                           "how": "fr_pack to the host buffer, then fr_unpack_verify from it, with the flips"}}
