@@ -233,6 +233,24 @@ fr_status fr_restore(fr_plan src, fr_plan dst, void* staging, uint64_t staging_b
                      uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev, void* stream_src,
                      void* stream_dst);
 
+/* Restoration from several healthy replicas at once, each sending a share of
+ * the chunks (the partitioned form of the restore: with R replicas alive,
+ * each packs about 1/R of the state).  Batch b of the plans is packed by
+ * replica src[b % n_src] on streams_src[b % n_src] (streams_src may be NULL:
+ * the legacy default stream for all) and unpacked and verified into `dst` on
+ * `stream_dst` as soon as it is packed; retry round r re-sends the failing
+ * chunks from replica r % n_src; then the still-failing chunks are listed as
+ * fr_unpack_verify does.  `fp_dst_dev` (or NULL) receives the restored
+ * state's fingerprint table.  Every source plan must describe the same layout
+ * and batch count as `dst` (else FR_ERR_PLAN_MISMATCH).  Sources on distinct
+ * streams pack concurrently; sharing a stream is correct, only serial.  All
+ * work is ordered before later work on `stream_dst`.
+ * Errors: FR_ERR_INVALID_ARG, FR_ERR_PLAN_MISMATCH, FR_ERR_ALIGNMENT,
+ * FR_ERR_BUFFER_TOO_SMALL, FR_ERR_CUDA. */
+fr_status fr_restore_multi(const fr_plan* src, uint32_t n_src, fr_plan dst, void* staging, uint64_t staging_bytes,
+                           uint32_t max_retries, uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev,
+                           fr_fp* fp_dst_dev, void* const* streams_src, void* stream_dst);
+
 /* ---------------------------------------------------------------- sharded (ZeRO / FSDP) state */
 
 /* With ZeRO / FSDP every data-parallel rank keeps only a shard of the

@@ -749,6 +749,64 @@ fr_status fr_restore_fp(fr_plan src, fr_plan dst, void* staging, uint64_t stagin
   return e == cudaSuccess ? FR_OK : cuda_fail(e, "compaction kernel launch");
 }
 
+fr_status fr_restore_multi(const fr_plan* src, uint32_t n_src, fr_plan dst, void* staging, uint64_t staging_bytes,
+                           uint32_t max_retries, uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev,
+                           fr_fp* fp_dst_dev, void* const* streams_src, void* stream_dst) {
+  if (src == nullptr || n_src == 0) return invalid("no source plans");
+  if (dst == nullptr) return invalid("plan is null");
+  if (n_mismatch_dev == nullptr) return invalid("n_mismatch_dev is null");
+  if (cap > 0 && mismatch_dev == nullptr) return invalid("mismatch_dev is null");
+  for (uint32_t i = 0; i < n_src; ++i) {
+    if (src[i] == nullptr) return invalid("a source plan is null");
+    fr_status st = check_same_layout(src[i], dst);
+    if (st != FR_OK) return st;
+  }
+  DeviceGuard g(dst->device);
+  if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
+  cudaStream_t sd = static_cast<cudaStream_t>(stream_dst);
+  auto ss = [&](uint32_t i) { return static_cast<cudaStream_t>(streams_src ? streams_src[i] : nullptr); };
+  if (dst->n_chunks == 0) {
+    cudaError_t e = cudaMemsetAsync(n_mismatch_dev, 0, sizeof(uint64_t), sd);
+    return e == cudaSuccess ? FR_OK : cuda_fail(e, "cudaMemsetAsync");
+  }
+  fr_status st = check_packed_buffer(dst, staging, staging_bytes);
+  if (st != FR_OK) return st;
+  uint8_t* buf = static_cast<uint8_t*>(staging);
+  FpEntry* fd = reinterpret_cast<FpEntry*>(fp_dst_dev);
+  const int umode = fd ? kModeUnpackFp : kModeUnpack;
+  const Decomp& DD = batch_for(dst, umode);
+  cudaError_t e;
+  // Batch b is packed by replica b mod n_src on its own stream and unpacked
+  // on the receiver's stream as soon as it is packed.
+  for (uint32_t b = 0; b < dst->n_batches; ++b) {
+    const uint32_t i = b % n_src;
+    st = run_batches(src[i], batch_for(src[i], kModePack), kModePack, buf, nullptr, b, b + 1, ss(i));
+    if (st != FR_OK) return st;
+    if ((e = cudaEventRecord(src[i]->events[b], ss(i))) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    if ((e = cudaStreamWaitEvent(sd, src[i]->events[b], 0)) != cudaSuccess)
+      return cuda_fail(e, "cudaStreamWaitEvent");
+    st = run_batches(dst, DD, umode, buf, fd, b, b + 1, sd);
+    if (st != FR_OK) return st;
+  }
+  // Retries: round r re-sends the failing chunks from replica r mod n_src.
+  for (uint32_t r = 0; r < max_retries; ++r) {
+    uint64_t failing = 0;
+    const uint32_t i = r % n_src;
+    st = resend_failed(src[i], dst, buf, ss(i), sd, &failing, nullptr, fd);
+    if (st != FR_OK) return st;
+    if (failing == 0) break;
+  }
+  // Everything queued on every replica's stream is ordered before what
+  // follows on the receiver's stream.
+  for (uint32_t i = 0; i < n_src; ++i) {
+    cudaEvent_t ev_end = src[i]->events[src[i]->n_batches];
+    if ((e = cudaEventRecord(ev_end, ss(i))) != cudaSuccess || (e = cudaStreamWaitEvent(sd, ev_end, 0)) != cudaSuccess)
+      return cuda_fail(e, "order the end of the restore");
+  }
+  e = launch_compact_flags(dst->d_flags, dst->n_chunks, mismatch_dev, cap, n_mismatch_dev, dst->d_status, sd);
+  return e == cudaSuccess ? FR_OK : cuda_fail(e, "compaction kernel launch");
+}
+
 fr_status fr_resend(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint64_t* n_resent,
                     void* stream_src, void* stream_dst) {
   return fr_resend_fp(src, dst, staging, staging_bytes, n_resent, nullptr, nullptr, stream_src, stream_dst);

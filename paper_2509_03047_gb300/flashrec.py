@@ -77,6 +77,8 @@ def _load() -> ctypes.CDLL:
     L.fr_unpack_verify_fp.argtypes = [vp, vp, u64, vp, u64, vp, vp, vp]
     L.fr_restore_fp.argtypes = [vp, vp, vp, u64, u32, vp, u64, vp, vp, vp, vp, vp]
     L.fr_resend_fp.argtypes = [vp, vp, vp, u64, u64p, vp, vp, vp, vp]
+    L.fr_restore_multi.argtypes = [ctypes.POINTER(vp), u32, vp, vp, u64, u32, vp, u64, vp, vp,
+                                   ctypes.POINTER(vp), vp]
     L.fr_status_str.argtypes = [ctypes.c_int]
     L.fr_status_str.restype = ctypes.c_char_p
     L.fr_last_error.argtypes = []
@@ -86,7 +88,7 @@ def _load() -> ctypes.CDLL:
                  "fr_unpack_verify", "fr_diff", "fr_sync_status", "fr_version", "fr_fingerprint_static",
                  "fr_plan_create_batched", "fr_plan_batch", "fr_pack_batch", "fr_unpack_verify_batch",
                  "fr_unpack_collect", "fr_resend", "fr_restore", "fr_shard_pieces", "fr_pack_fp", "fr_unpack_verify_fp",
-                 "fr_restore_fp", "fr_resend_fp"]:
+                 "fr_restore_fp", "fr_resend_fp", "fr_restore_multi"]:
         getattr(L, name).restype = ctypes.c_int
     return L
 
@@ -233,6 +235,21 @@ def fr_resend_fp(src_plan, dst_plan, staging: torch.Tensor, fp_src: Optional[tor
                             ctypes.byref(n), _table_ptr(fp_src), _table_ptr(fp_dst), _stream(stream_src),
                             _stream(stream_dst)), "fr_resend_fp")
     return n.value
+
+
+def fr_restore_multi(src_plans, dst_plan, staging: torch.Tensor, max_retries: int, mismatch: Optional[torch.Tensor],
+                     count: torch.Tensor, fp_dst: Optional[torch.Tensor] = None, streams_src=None,
+                     stream_dst=None) -> None:
+    """Restore `dst_plan` from several replicas, batch b packed by replica b % len(src_plans)."""
+    n = len(src_plans)
+    plans = (ctypes.c_void_p * n)(*[p for p in src_plans])
+    streams = None
+    if streams_src is not None:
+        streams = (ctypes.c_void_p * n)(*[_stream(x) for x in streams_src])
+    cap = 0 if mismatch is None else mismatch.numel()
+    _check(lib.fr_restore_multi(plans, n, dst_plan, staging.data_ptr() if staging.numel() else None, staging.numel(),
+                                max_retries, mismatch.data_ptr() if cap else None, cap, count.data_ptr(),
+                                _table_ptr(fp_dst), streams, _stream(stream_dst)), "fr_restore_multi")
 
 
 def fr_plan_info(plan):
