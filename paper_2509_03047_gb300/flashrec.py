@@ -401,6 +401,25 @@ class Plan:
         n = int(count.item())
         return mismatch[: min(n, mismatch.numel())], n
 
+    def pack_fp(self, dst: Optional[torch.Tensor] = None, table: Optional[torch.Tensor] = None, stream=None):
+        """fr_pack_fp: returns (packed buffer, this state's fingerprint table)."""
+        dst = self.new_packed() if dst is None else dst
+        table = self.new_table() if table is None else table
+        fr_pack_fp(self.handle, dst, table, stream)
+        return dst, table
+
+    def unpack_verify_fp(self, src: torch.Tensor, table: Optional[torch.Tensor] = None, cap: Optional[int] = None,
+                         stream=None):
+        """fr_unpack_verify_fp: returns (mismatch ids, count, the restored state's
+        fingerprint table) after a sync."""
+        cap = self.n_chunks if cap is None else cap
+        mismatch = torch.empty(max(cap, 1), dtype=torch.int32, device=self.device)[:cap]
+        count = torch.empty(1, dtype=torch.int64, device=self.device)
+        table = self.new_table() if table is None else table
+        fr_unpack_verify_fp(self.handle, src, mismatch, count, table, stream)
+        n = int(count.item())
+        return mismatch[: min(n, mismatch.numel())], n, table
+
     def sync_status(self, stream=None) -> int:
         return fr_sync_status(self.handle, stream)
 

@@ -147,3 +147,14 @@ def test_resend_fp_rewrites_the_resent_entries():
     assert _same(st, dst_t)
     assert torch.equal(fa, src.fingerprint())
     assert torch.equal(fb, fa)
+
+
+def test_plan_methods_for_the_fused_calls():
+    _, st, chunk = _case("tiny")
+    a = fr.Plan(st, chunk)
+    packed, ta = a.pack_fp()
+    assert torch.equal(ta, a.fingerprint()) and torch.equal(packed, a.pack())
+    out = _fresh(st)
+    b = fr.Plan(out, chunk)
+    ids, n, tb = b.unpack_verify_fp(packed)
+    assert n == 0 and torch.equal(ta, tb) and _same(st, out)
