@@ -158,3 +158,25 @@ def test_plan_methods_for_the_fused_calls():
     b = fr.Plan(out, chunk)
     ids, n, tb = b.unpack_verify_fp(packed)
     assert n == 0 and torch.equal(ta, tb) and _same(st, out)
+
+
+@pytest.mark.parametrize("name", ["l70b_tp8pp4", "zero_frag"])
+def test_fused_calls_at_full_size(name):
+    """The bench's workloads at full size, with its flips: the fused tables
+    are bit-identical to fr_fingerprint's (sampled against the oracle in
+    test_gpu_parity.py), the failure list to the plain call's."""
+    cfg = synth.get_config(name)
+    st = synth.make_state(cfg, "cuda")
+    synth.inject_nonfinite(cfg, st)
+    a = fr.Plan(st, cfg.chunk_bytes)
+    packed, ta = a.pack_fp()
+    assert torch.equal(ta, a.fingerprint())
+    flips = synth.flip_positions(a.packed_bytes, max(cfg.flips, 10), cfg.seed)
+    synth.apply_flips(packed, flips)
+    out = [torch.empty_like(t) for t in st]
+    b = fr.Plan(out, cfg.chunk_bytes)
+    ids, n, tb = b.unpack_verify_fp(packed)
+    assert np.array_equal(ids.cpu().numpy().astype(np.int64), expected_mismatch(_chunks(st, cfg.chunk_bytes), flips))
+    assert torch.equal(tb, b.fingerprint())
+    d, k = fr.diff(ta, tb)
+    assert k >= 1 and set(d.cpu().numpy().tolist()) <= set(ids.cpu().numpy().tolist())
