@@ -37,7 +37,51 @@ constexpr unsigned kFull = 0xFFFFFFFFu;
 
 __device__ const ByteTable g_byte = make_byte_table();
 __device__ const PowTables g_pow = make_pow_tables();
-__device__ const TailMuls g_tail = make_tail_muls();
+// Byte tables for multiplying by the constants x^(32 * 2^k), k = 0..6
+// (x^32 ... x^2048): the shuffle trees that join 4-byte header words and
+// 16-byte tail pieces lane by lane.
+struct ConstMulTables {
+  ByteTables4 m[7];
+};
+__host__ __device__ constexpr ConstMulTables make_const_mul_tables() {
+  ConstMulTables t{};
+  for (int k = 0; k < 7; ++k) t.m[k] = make_mul_tables(gf_xpow(32ull << k));
+  return t;
+}
+__device__ const ConstMulTables g_cmul = make_const_mul_tables();
+
+// a * x^(32 * 2^k) mod P.
+__device__ __forceinline__ uint32_t mul_x32k(int k, uint32_t a) {
+  const ByteTables4& T = g_cmul.m[k];
+  return (__ldg(&T.t[0][a & 255u]) ^ __ldg(&T.t[1][(a >> 8) & 255u])) ^
+         (__ldg(&T.t[2][(a >> 16) & 255u]) ^ __ldg(&T.t[3][a >> 24]));
+}
+
+// Joins the raw CRCs v of lanes 0..2^levels-1, lane l holding piece l of
+// 4 * 2^first bytes each, in lane order: lane 0 ends with raw(piece 0 || ... ).
+__device__ __forceinline__ uint32_t join_lanes(uint32_t v, int first, int levels) {
+  for (int j = 0; j < levels; ++j) {
+    const uint32_t o = __shfl_down_sync(kFull, v, 1u << j);
+    v = mul_x32k(first + j, v) ^ o;
+  }
+  return v;
+}
+
+// CRC-32C of the 60 header bytes given as 15 words, computed by lanes 1..15
+// (lane l CRCs word l-1; lane 0 is a leading zero word, which leaves a raw
+// CRC run from zero unchanged) and joined in a 4-level tree; all lanes return
+// it.  `T` is the byte table.
+__device__ __forceinline__ uint32_t header_crc(const uint32_t* T, const uint32_t h[15], uint32_t lane) {
+  uint32_t w = 0;
+#pragma unroll
+  for (int k = 0; k < 15; ++k) w = (lane == static_cast<uint32_t>(k + 1)) ? h[k] : w;
+  uint32_t r = 0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) r = T[(r ^ (w >> (8 * j))) & 0xFFu] ^ (r >> 8);
+  const uint32_t raw = join_lanes(lane < 16 ? r : 0u, 0, 4);
+  constexpr uint32_t kHeaderXor = gf_mulmod(0xFFFFFFFFu, gf_xpow(8 * 60)) ^ 0xFFFFFFFFu;
+  return __shfl_sync(kFull, raw, 0) ^ kHeaderXor;
+}
 
 // a * b mod P, both variable.
 __device__ __forceinline__ uint32_t gmul(uint32_t a, uint32_t b) {
@@ -208,6 +252,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
     float th = 0.0f, tl = 0.0f;  // the tail's sum of squares, as a float pair
     double tdx = 0.0;            // and its rare fp64 part
     uint32_t nf_tail = 0;
+    uint32_t tail_raw = 0;
     const int32_t e1 = static_cast<int32_t>(tail) - 16 * (31 - static_cast<int32_t>(lane));
     if (e1 > 0) {
       const uint32_t b1 = static_cast<uint32_t>(e1);
@@ -228,8 +273,12 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
           }
         }
       }
-      raw ^= gmul(r, g_tail.m[lane]);
+      tail_raw = r;
     }
+    // lane l's piece ends 16 * (31 - l) bytes before the tail's end: join the
+    // 32 pieces in lane order; lane 0 holds the tail's raw CRC
+    tail_raw = join_lanes(tail_raw, 2, 5);
+    if (lane == 0) raw ^= tail_raw;
 #pragma unroll
     for (int m = 16; m >= 1; m >>= 1) {
       raw ^= __shfl_xor_sync(kFull, raw, m);
@@ -245,8 +294,9 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
 
     // ---- 3. preset and final XOR
     const uint32_t crc = raw ^ (p.crc_xor ? p.crc_xor[c] : (shift_bytes(0xFFFFFFFFu, cd.len) ^ 0xFFFFFFFFu));
-    const double sumsq = sq_rec + sq_tail;  // lane 0 holds the fixed-order sums
-    const uint32_t nonfinite = nf_rec + nf_tail;
+    // lane 0 holds the fixed-order sums and counts: every lane gets them
+    const double sumsq = __shfl_sync(kFull, sq_rec + sq_tail, 0);
+    const uint32_t nonfinite = __shfl_sync(kFull, nf_rec + nf_tail, 0);
 
     const uint64_t pad_begin = cd.payload_off + cd.len;
     const uint64_t pad_end = cd.payload_off + align_up(cd.len, kPayloadAlign);
@@ -265,8 +315,8 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
       }
     }
     if (MODE == kModePack) {
-      if (lane == 0) {
-        uint32_t h[16];
+      {
+        uint32_t h[15];
         const uint64_t sbits = static_cast<uint64_t>(__double_as_longlong(sumsq));
         h[0] = kMagic;
         h[1] = kVersion | (cd.dtype << 16);
@@ -283,40 +333,35 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
         h[12] = static_cast<uint32_t>(sbits);
         h[13] = static_cast<uint32_t>(sbits >> 32);
         h[14] = nonfinite;
-        uint32_t r = 0xFFFFFFFFu;
-        for (int i = 0; i < 15; ++i)
-          for (int j = 0; j < 4; ++j) r = crc_byte(T, r, (h[i] >> (8 * j)) & 0xFFu);
-        h[15] = r ^ 0xFFFFFFFFu;
-        uint4* dst = reinterpret_cast<uint4*>(p.packed + c * kHeaderBytes);
-        for (int q = 0; q < 4; ++q) dst[q] = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+        const uint32_t hcrc = header_crc(T, h, lane);
+        if (lane == 0) {
+          uint4* dst = reinterpret_cast<uint4*>(p.packed + c * kHeaderBytes);
+          for (int q = 0; q < 3; ++q) dst[q] = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+          dst[3] = make_uint4(h[12], h[13], h[14], hcrc);
+        }
       }
       for (uint64_t j = pad_begin + lane; j < pad_end; j += 32) p.packed[j] = 0;
       if (last)
         for (uint64_t j = table_end + lane * 16u; j < gap_end; j += 512)
           *reinterpret_cast<uint4*>(p.packed + j) = make_uint4(0, 0, 0, 0);
     } else if (mode_unpacks(MODE)) {  // unpack + verify
-      bool bad = false;
-      if (lane == 0) {
-        const uint4* src = reinterpret_cast<const uint4*>(p.packed + c * kHeaderBytes);
-        uint32_t h[16];
-        for (int q = 0; q < 4; ++q) {
-          const uint4 v = src[q];
-          h[4 * q] = v.x;
-          h[4 * q + 1] = v.y;
-          h[4 * q + 2] = v.z;
-          h[4 * q + 3] = v.w;
-        }
-        uint32_t r = 0xFFFFFFFFu;
-        for (int i = 0; i < 15; ++i)
-          for (int j = 0; j < 4; ++j) r = crc_byte(T, r, (h[i] >> (8 * j)) & 0xFFu);
-        bad = (h[15] != (r ^ 0xFFFFFFFFu)) || h[0] != kMagic || (h[1] & 0xFFFFu) != kVersion ||
-              (h[1] >> 16) != cd.dtype || h[2] != static_cast<uint32_t>(c) ||
-              h[3] != static_cast<uint32_t>(c >> 32) || h[4] != cd.tensor_idx ||
-              h[6] != static_cast<uint32_t>(cd.tensor_off) || h[7] != static_cast<uint32_t>(cd.tensor_off >> 32) ||
-              h[8] != static_cast<uint32_t>(cd.len) || h[9] != static_cast<uint32_t>(cd.len >> 32) ||
-              h[10] != static_cast<uint32_t>(cd.payload_off) ||
-              h[11] != static_cast<uint32_t>(cd.payload_off >> 32) || h[5] != crc;
+      // every lane reads the (same) header and checks it against the plan
+      const uint4* src = reinterpret_cast<const uint4*>(p.packed + c * kHeaderBytes);
+      uint32_t h[16];
+      for (int q = 0; q < 4; ++q) {
+        const uint4 v = src[q];
+        h[4 * q] = v.x;
+        h[4 * q + 1] = v.y;
+        h[4 * q + 2] = v.z;
+        h[4 * q + 3] = v.w;
       }
+      const uint32_t hcrc = header_crc(T, h, lane);
+      bool bad = (h[15] != hcrc) || h[0] != kMagic || (h[1] & 0xFFFFu) != kVersion || (h[1] >> 16) != cd.dtype ||
+                 h[2] != static_cast<uint32_t>(c) || h[3] != static_cast<uint32_t>(c >> 32) ||
+                 h[4] != cd.tensor_idx || h[6] != static_cast<uint32_t>(cd.tensor_off) ||
+                 h[7] != static_cast<uint32_t>(cd.tensor_off >> 32) || h[8] != static_cast<uint32_t>(cd.len) ||
+                 h[9] != static_cast<uint32_t>(cd.len >> 32) || h[10] != static_cast<uint32_t>(cd.payload_off) ||
+                 h[11] != static_cast<uint32_t>(cd.payload_off >> 32) || h[5] != crc;
       for (uint64_t j = pad_begin + lane; j < pad_end; j += 32)
         if (p.packed[j] != 0) bad = true;
       if (last)

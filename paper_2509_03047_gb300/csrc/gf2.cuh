@@ -150,15 +150,4 @@ inline uint32_t host_xpow8(uint64_t n) {
 // crc = raw ^ crc_xor_term(n), raw being the CRC register run from zero.
 inline uint32_t host_crc_xor_term(uint64_t n) { return gf_mulmod(0xFFFFFFFFu, host_xpow8(n)) ^ 0xFFFFFFFFu; }
 
-// Shifts of the 16-byte lane pieces of a chunk tail laid out against its end:
-// lane l's piece is followed by 16 * (31 - l) bytes.
-struct TailMuls {
-  uint32_t m[32];
-};
-__host__ __device__ constexpr TailMuls make_tail_muls() {
-  TailMuls t{};
-  for (int l = 0; l < 32; ++l) t.m[l] = gf_xpow(128ull * (31 - l));
-  return t;
-}
-
 }  // namespace frk
