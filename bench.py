@@ -360,7 +360,16 @@ def run_flashrec(args):
     # ---- end to end through the C ABI with the transfer buffer in pinned host memory
     e2e = None
     if not args.no_e2e:
-        host_buf = plan_s.new_packed(pinned=True)
+        try:
+            host_buf = plan_s.new_packed(pinned=True)
+        except RuntimeError as exc:  # pinning P bytes per rank can fail on a crowded host
+            host_buf = None
+            e2e = {"unavailable": "pinned host buffer of %d bytes: %s" % (P, str(exc).splitlines()[0])}
+        # every rank takes the leg (it has collectives) only if every rank could pin
+        if max_over_ranks(0.0 if host_buf is not None else 1.0, dev) > 0.0 and host_buf is not None:
+            e2e = {"unavailable": "another rank could not pin its host buffer"}
+            host_buf = None
+    if not args.no_e2e and host_buf is not None:
         # (a) the pipelined restore: batches packed on the replica's stream and
         # unpacked on the receiver's stream as soon as each is packed, so both
         # directions of the host link work at once; one re-send round
