@@ -179,7 +179,7 @@ def _rank_main(rank: int, world: int, host: str, port: int, n_steps: int, fail_s
 
 def simulate(world: int, dp_groups: Sequence[Sequence[int]], n_steps: int, fail_rank: int, fail_step: int,
              fail_phase: str, step_time: float = 0.02, timeout: float = 60.0, fail_mode: str = "exit",
-             heartbeat_timeout: float = 1.0):
+             heartbeat_timeout: float = 5.0):
     """Run `world` CPU ranks; rank `fail_rank` dies ("exit") or goes silent
     ("hang") in `fail_phase` of step `fail_step`.  Returns (decision, {rank:
     updates held when stopped})."""

@@ -82,7 +82,7 @@ def test_heartbeat_timeout_declares_a_silent_rank_failed():
 @pytest.mark.parametrize("phase,resume", [("forward_backward", 2), ("optimizer", 3)])
 def test_simulated_hang_is_found_by_its_silent_heartbeat(phase, resume):
     decision, held = st.simulate(world=4, dp_groups=GROUPS, n_steps=6, fail_rank=2, fail_step=2, fail_phase=phase,
-                                 fail_mode="hang", heartbeat_timeout=0.5)
+                                 fail_mode="hang", heartbeat_timeout=2.0)
     assert decision.restore == [2] and decision.source == {2: 0}
     assert decision.resume_step == resume and decision.phase == phase
     assert set(held.values()) == {resume}
