@@ -357,6 +357,44 @@ def run_flashrec(args):
              "how": "fr_pack_fp -> flips -> fr_unpack_verify_fp -> fr_diff: both fingerprint tables come out of "
                     "the pack and unpack sweeps; same outputs as the step above"}
 
+    # ---- optionally, the fused step captured once in a CUDA graph and replayed
+    # (the calls only enqueue kernels, so small states can shed launch overhead)
+    graph = None
+    if args.graph:
+        gs = torch.cuda.Stream(device=dev)
+
+        def graph_body():
+            fr.fr_pack_fp(plan_s.handle, packed, tab_s, gs)
+            fr.fr_unpack_verify_fp(plan_d.handle, packed, mism, nmis, tab_d, gs)
+            fr.fr_diff(tab_s, tab_d, C, div, ndiv, gs)
+
+        gs.wait_stream(stream)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=gs):
+            graph_body()
+        for _ in range(args.warmup):
+            g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        g_ms = e0.elapsed_time(e1) / args.steps
+        e0.record(stream)
+        for _ in range(args.steps):
+            fr.fr_pack_fp(plan_s.handle, packed, tab_s, stream)
+            fr.fr_unpack_verify_fp(plan_d.handle, packed, mism, nmis, tab_d, stream)
+            fr.fr_diff(tab_s, tab_d, C, div, ndiv, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        eager_ms = e0.elapsed_time(e1) / args.steps
+        graph = {"ms_per_step": round(g_ms, 4), "eager_ms_per_step": round(eager_ms, 4),
+                 "how": "fr_pack_fp -> fr_unpack_verify_fp -> fr_diff captured once in a CUDA graph and "
+                        "replayed back to back (no flips), against the same calls launched eagerly"}
+        del g
+
     # ---- end to end through the C ABI with the transfer buffer in pinned host memory
     e2e = None
     if not args.no_e2e:
@@ -473,7 +511,8 @@ def run_flashrec(args):
                           "l2": "inputs larger than L2 (state %.1f GB vs 129 MB L2); no flush" % (S / 1e9),
                           "parallelism": "replicas only (%d independent rank%s)" % (ws, "s" if ws > 1 else ""),
                           "value_def": "4 sweeps x state bytes / step time"},
-               "calls": calls, "roofline": roofline, "fused_step": fused, "e2e": e2e, "cpu_baseline": cpu,
+               "calls": calls, "roofline": roofline, "fused_step": fused, "graph_step": graph, "e2e": e2e,
+               "cpu_baseline": cpu,
                "gpu_launches": launches_per_step * args.steps, "clocks": clk}
         print(json.dumps(out))
     plan_s.close()
@@ -590,6 +629,7 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-gb", type=float, default=1.0)
+    ap.add_argument("--graph", action="store_true", help="also time the fused step replayed from a CUDA graph")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "flashrec":
         ap.error("at least 3 warm-up steps")
