@@ -369,3 +369,35 @@ def test_zero_frag_full_size_sampled_and_diff():
     d, k = fr.diff(table, tm)
     assert k == cfg.diff_chunks == 100
     assert np.array_equal(d.cpu().numpy().astype(np.int64), ids)
+
+
+def test_chunk_larger_than_4_gib():
+    """One fp32 tensor of 6 GiB + 37 elements in 5 GiB chunks: lengths,
+    offsets, shift exponents and header fields beyond 32 bits.  Fingerprint
+    against the oracle, headers byte-exact against the oracle's (with the
+    GPU's sums), and a clean round trip."""
+    n = (6 << 30) // 4 + 37
+    g = torch.Generator(device="cuda")
+    g.manual_seed(17)
+    t = torch.randn(n, generator=g, device="cuda")
+    t[123456789] = float("nan")
+    t[n - 5] = float("inf")
+    chunk = 5 << 30
+    p = fr.Plan([t], chunk)
+    assert p.n_chunks == 2
+    table = table_np(p.fingerprint())
+    host = host_bytes([t])
+    want = oracle.fingerprint(host, [fr.FR_DT_F32], chunk)
+    assert_tables_match(table, want, "6 GiB tensor")
+    packed = p.pack()
+    chunks, _ = oracle.plan([host[0].size], [fr.FR_DT_F32], chunk)
+    head = packed[: 2 * 64].cpu().numpy()
+    for c in range(2):
+        fp = (int(want["crc32c"][c]), int(want["nonfinite"][c]), float(table["sumsq"][c]))
+        assert np.array_equal(head[64 * c: 64 * c + 64], np.frombuffer(oracle.header(chunks[c], c, fp), dtype=np.uint8))
+    del host
+    out = torch.empty_like(t)
+    q = fr.Plan([out], chunk)
+    ids, k = q.unpack_verify(packed)
+    assert k == 0
+    assert torch.equal(out.view(torch.int32), t.view(torch.int32))
