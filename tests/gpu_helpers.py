@@ -123,3 +123,28 @@ def compare_full(tensors, chunk_bytes, flips=None):
         assert np.array_equal(g, w), "restored tensor %d differs" % i
     assert got["status"] == fr.FR_OK
     return got, want
+
+
+def odd_tensors(seed=0, offset=0):
+    """Tensors of awkward sizes (empty, a few bytes, just over and under 512-byte
+    blocks and 16 KiB segments, several MiB), each a view starting `offset`
+    bytes into its buffer where the element size allows (else aligned)."""
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    sizes = [(torch.float32, 0), (torch.bfloat16, 6), (torch.float32, 4), (torch.float32, 20),
+             (torch.uint8, 13), (torch.bfloat16, 1000), (torch.float32, 4096), (torch.float32, 4100),
+             (torch.bfloat16, 8194), (torch.float32, 3 * 1024 + 12), (torch.float32, 512),
+             (torch.float32, 511 * 4), (torch.bfloat16, 70000), (torch.float32, 1 << 20),
+             (torch.float32, (1 << 20) + 516), (torch.uint8, 100003), (torch.bfloat16, 262144 * 2 + 2)]
+    out = []
+    for dt, nbytes in sizes:
+        if dt == torch.uint8:
+            base = torch.randint(0, 256, (nbytes + 16,), generator=g, device="cuda", dtype=torch.uint8)
+            out.append(base[offset:offset + nbytes])
+            continue
+        esz = 4 if dt == torch.float32 else 2
+        n = nbytes // esz
+        eo = offset // esz if offset % esz == 0 else 0
+        base = torch.randn(n + 8, generator=g, device="cuda", dtype=torch.float32).to(dt)
+        out.append(base[eo:eo + n])
+    return out

@@ -8,7 +8,7 @@ import torch
 
 from paper_2509_03047_gb300 import synth
 
-from gpu_helpers import expected_mismatch, table_np
+from gpu_helpers import assert_tables_match, expected_mismatch, odd_tensors, table_np
 
 pytestmark = pytest.mark.gpu
 
@@ -97,6 +97,41 @@ def test_unpack_verify_fp_equals_unpack_then_fingerprint(name):
     assert _same(a_t, b_t)
     # the table is the fingerprint of what was written, failing chunks included
     assert torch.equal(got_table, b.fingerprint())
+
+
+@pytest.mark.parametrize("offset,chunk", [(0, 4), (0, 12), (0, 1000), (0, 64 * KiB), (2, 4096), (4, 12288),
+                                          (8, 100)])
+def test_fused_calls_on_odd_sizes_and_views(offset, chunk):
+    """Every piece shape the fused sweeps meet -- sub-block tails, chunks of a
+    few bytes, tensors shorter than a lane's unit, misaligned views -- against
+    the plain calls and, for the tables, the oracle."""
+    st = odd_tensors(5, offset)
+    src = fr.Plan(st, chunk)
+    want_table, want_packed = src.fingerprint(), src.pack()
+    packed = torch.full_like(want_packed, 0xCC)
+    ta = torch.full_like(want_table, 0xEE)
+    fr.fr_pack_fp(src.handle, packed, ta)
+    torch.cuda.synchronize()
+    assert torch.equal(packed, want_packed) and torch.equal(ta, want_table)
+    chunks = _chunks(st, chunk)
+    host = [t.contiguous().view(torch.uint8).cpu().numpy().reshape(-1) for t in st]
+    want_fp = oracle.fingerprint(host, [fr.fr_dtype_of(t) for t in st], chunk)
+    assert_tables_match(table_np(ta), want_fp, "pack_fp")
+
+    flips = synth.flip_positions(src.packed_bytes, 5, seed=offset + chunk)
+    synth.apply_flips(packed, flips)
+    dst_t = _fresh(st)
+    dst = fr.Plan(dst_t, chunk)
+    ids = torch.empty(dst.n_chunks, dtype=torch.int32, device="cuda")
+    cnt = torch.empty(1, dtype=torch.int64, device="cuda")
+    tb = torch.full_like(want_table, 0xDD)
+    fr.fr_unpack_verify_fp(dst.handle, packed, ids, cnt, tb)
+    n = int(cnt.item())
+    assert np.array_equal(ids[:n].cpu().numpy().astype(np.int64), expected_mismatch(chunks, flips))
+    assert torch.equal(tb, dst.fingerprint())
+    # chunks whose payload took no flip are restored bit-exactly, with equal entries
+    d, k = fr.diff(ta, tb)
+    assert set(d.cpu().tolist()) <= set(ids[:n].cpu().tolist())
 
 
 @pytest.mark.parametrize("where,n_batches", [("device", 1), ("device", 7), ("pinned", 5)])

@@ -14,7 +14,7 @@ import torch
 import oracle
 from paper_2509_03047_gb300 import synth
 
-from gpu_helpers import (assert_tables_match, compare_full, expected_mismatch, host_bytes,
+from gpu_helpers import (assert_tables_match, compare_full, expected_mismatch, host_bytes, odd_tensors,
                          payload_flip_chunks, run_full, table_np)
 
 pytestmark = pytest.mark.gpu
@@ -57,36 +57,14 @@ def test_gpt2_small_whole_state_clean_roundtrip():
         assert torch.equal(a.view(torch.uint8), b.view(torch.uint8))
 
 
-def _odd_tensors(seed=0, offset=0):
-    g = torch.Generator(device="cuda")
-    g.manual_seed(seed)
-    sizes = [(torch.float32, 0), (torch.bfloat16, 6), (torch.float32, 4), (torch.float32, 20),
-             (torch.uint8, 13), (torch.bfloat16, 1000), (torch.float32, 4096), (torch.float32, 4100),
-             (torch.bfloat16, 8194), (torch.float32, 3 * 1024 + 12), (torch.float32, 512),
-             (torch.float32, 511 * 4), (torch.bfloat16, 70000), (torch.float32, 1 << 20),
-             (torch.float32, (1 << 20) + 516), (torch.uint8, 100003), (torch.bfloat16, 262144 * 2 + 2)]
-    out = []
-    for dt, nbytes in sizes:
-        if dt == torch.uint8:
-            base = torch.randint(0, 256, (nbytes + 16,), generator=g, device="cuda", dtype=torch.uint8)
-            out.append(base[offset:offset + nbytes])
-            continue
-        esz = 4 if dt == torch.float32 else 2
-        n = nbytes // esz
-        eo = offset // esz if offset % esz == 0 else 0
-        base = torch.randn(n + 8, generator=g, device="cuda", dtype=torch.float32).to(dt)
-        out.append(base[eo:eo + n])
-    return out
-
-
 @pytest.mark.parametrize("chunk", [4, 12, 100, 512, 1000, 4096, 64 * KiB, 1 * MiB])
 def test_adversarial_sizes_and_chunks(chunk):
-    compare_full(_odd_tensors(1), chunk)
+    compare_full(odd_tensors(1), chunk)
 
 
 @pytest.mark.parametrize("offset", [4, 8, 2])
 def test_misaligned_views(offset):
-    ts = _odd_tensors(2, offset)
+    ts = odd_tensors(2, offset)
     assert any(t.data_ptr() % 16 for t in ts if t.numel())
     compare_full(ts, 4096)
     compare_full(ts, 64 * KiB)
