@@ -55,7 +55,7 @@ struct Decomp {
   WarpDesc* d_warps = nullptr;
   uint32_t* d_lists = nullptr;
   uint64_t* d_rec_nblk = nullptr;
-  uint32_t* d_rec_mul = nullptr;  // per record: x^(8 * bytes after it in its chunk)
+  uint32_t* d_rec_mul = nullptr;  // per record: x^(8 * bytes after it in its chunk's body)
   Record* d_recs = nullptr;
 };
 
@@ -244,7 +244,7 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
             if (d.n_recs == 0) d.first_rec = static_cast<uint32_t>(rec_nblk.size());
             d.n_recs += 1;
             rec_nblk.push_back(n);
-            rec_mul.push_back(host_xpow8(d.len - (bb - d.blk_begin + n) * kBlockBytes));
+            rec_mul.push_back(host_xpow8((end - bb - n) * kBlockBytes));
             bb += n;
             if (bb == end) ++j;
           }

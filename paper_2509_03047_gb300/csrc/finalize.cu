@@ -3,13 +3,17 @@
 //
 // The sweep kernel leaves one record per piece (the part of a chunk body one
 // warp covered).  Here one warp per chunk:
-//   1. shifts each record's raw CRC to its position in the chunk and XORs them
-//      (raw(A||B) = raw(A) * x^(8|B|) ^ raw(B)), adds the records' non-finite
-//      counts, and adds the body's 16 KiB segment sums of squares in an order
-//      fixed by segment index (so the result does not depend on the plan);
-//   2. handles the chunk's tail (len % 512 bytes): lane l takes bytes
-//      [16l, 16l+16) of it, CRCs them a byte at a time, sums their squares in
-//      fp64, and copies them for pack/unpack;
+//   0. issues every load the chunk needs at once, after its descriptor;
+//   1. shifts each record's raw CRC to its position in the chunk's body and
+//      XORs them (raw(A||B) = raw(A) * x^(8|B|) ^ raw(B)), adds the records'
+//      non-finite counts, and adds the body's 16 KiB segment sums of squares
+//      in an order fixed by segment index (so the result does not depend on
+//      the plan);
+//   2. handles the chunk's tail (len % 512 bytes, if any): lane l takes the
+//      16 bytes ending 16 * (31 - l) bytes before its end, copies them for
+//      pack/unpack, sums their squares, and CRCs them a word at a time with
+//      the body's raw CRC folded into the tail's first word (which continues
+//      the body's CRC through the tail without shifting it);
 //   3. applies CRC-32C's preset and final XOR:
 //      crc = raw ^ 0xFFFFFFFF * x^(8 len) ^ 0xFFFFFFFF;
 //   4. fingerprint: writes the table entry; pack: writes the 64-byte header,
@@ -31,6 +35,9 @@ namespace frk {
 
 namespace {
 
+#ifndef FR_FIN_MINB
+#define FR_FIN_MINB 4  // finalize CTAs per SM (caps registers at 64: more chunks in flight)
+#endif
 constexpr int kFinWarps = 8;
 constexpr int kFinThreads = kFinWarps * 32;
 constexpr unsigned kFull = 0xFFFFFFFFu;
@@ -108,10 +115,6 @@ __device__ __forceinline__ uint32_t shift_bytes(uint32_t raw, uint64_t n) {
   return n ? gmul(raw, xpow8(n)) : raw;
 }
 
-__device__ __forceinline__ uint32_t crc_byte(const uint32_t* T, uint32_t r, uint32_t b) {
-  return T[(r ^ b) & 0xFFu] ^ (r >> 8);
-}
-
 // (hi, lo) += (bh, bl) as unevaluated float pairs: TwoSum of the high parts,
 // the low parts and the rounding error added in fp32.
 __device__ __forceinline__ void two_sum_pair(float& hi, float& lo, float bh, float bl) {
@@ -148,8 +151,19 @@ __device__ __forceinline__ void tail_elem(uint32_t dtype, uint32_t bits, uint32_
   }
 }
 
+// Adds one segment slot (see seg_value) to the float pair (hi, lo) or, in the
+// tagged fp64 form, to dx.
+__device__ __forceinline__ void add_slot(uint64_t bits, float& hi, float& lo, double& dx) {
+  if (bits >> 63)
+    dx += -__longlong_as_double(static_cast<long long>(bits));
+  else
+    two_sum_pair(hi, lo, __uint_as_float(static_cast<uint32_t>(bits >> 32)), __uint_as_float(static_cast<uint32_t>(bits)));
+}
+
+__device__ __forceinline__ void prefetch_l1(const void* q) { asm volatile("prefetch.global.L1 [%0];" ::"l"(q)); }
+
 template <int MODE>
-__global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p) {
+__global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(FinalizeParams p) {
   __shared__ uint32_t T[256];
   for (int i = threadIdx.x; i < 256; i += kFinThreads) T[i] = g_byte.t[i];
   __syncthreads();
@@ -158,6 +172,8 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
   for (uint64_t pos = p.c_begin + static_cast<uint64_t>(blockIdx.x) * kFinWarps + (threadIdx.x >> 5);
        pos < p.c_end; pos += stride) {
     const uint64_t c = p.ids ? p.ids[pos] : pos;
+    // the warp's next descriptor streams into L1 while this chunk is done
+    if (!p.ids && lane == 0 && pos + stride < p.c_end) prefetch_l1(p.chunks + pos + stride);
     const ChunkDesc cd = p.chunks[c];
     const uint64_t body = cd.len & ~static_cast<uint64_t>(kBlockBytes - 1);
     const uint32_t tail = static_cast<uint32_t>(cd.len - body);
@@ -165,17 +181,77 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
     // list mode: one record per chunk with a body, at the list position
     const uint64_t first_rec = p.ids ? pos : cd.first_rec;
     const int64_t n_recs = p.ids ? (body ? 1 : 0) : cd.n_recs;
+    const uint64_t n_seg = (body / kBlockBytes + kSegBlocks - 1) / kSegBlocks;  // (read only with values)
+    const bool rec_mul = p.rec_mul && !p.ids;
 
-    // ---- 1. records: each shifted by the bytes after it in the chunk -- a
-    // multiplier the plan precomputed, or (list mode, no-allocation entry)
-    // found here, last batch of 32 first so the byte count after each is known
+    // ---- 0. every load the chunk needs (records, segment sums, tail bytes,
+    // preset term, header and padding) is issued here, before any is used, so
+    // a chunk costs one memory latency after its descriptor
+    Record rec0{0u, 0u, 0.0};
+    uint32_t mul0 = 0;
+    if (rec_mul && lane < n_recs) {
+      rec0 = p.recs[first_rec + lane];
+      mul0 = p.rec_mul[first_rec + lane];
+    }
+    uint64_t slot0 = 0;
+    if (values && lane < n_seg) slot0 = reinterpret_cast<const uint64_t*>(p.segs + cd.seg_base)[lane];
+    const uint8_t* tsrc;
+    uint8_t* tdst = nullptr;
+    if (mode_unpacks(MODE)) {
+      tsrc = p.packed + cd.payload_off + body;
+      tdst = reinterpret_cast<uint8_t*>(cd.addr) + body;
+    } else {
+      tsrc = reinterpret_cast<const uint8_t*>(cd.addr) + body;
+      if (MODE == kModePack) tdst = p.packed + cd.payload_off + body;
+    }
+    // lane l takes the 16 tail bytes that end 16 * (31 - l) bytes before the
+    // tail's end, as four little-endian words; bytes before the tail read as
+    // zeros (leading zero bytes leave a raw CRC run from zero unchanged and
+    // add nothing to the sums), so the lane's shift is a constant
+    const int32_t e0 = static_cast<int32_t>(tail) - 16 * (32 - static_cast<int32_t>(lane));
+    uint32_t w[4] = {0u, 0u, 0u, 0u};
+    if (tail != 0) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        if (e0 + j >= 0) w[j >> 2] |= static_cast<uint32_t>(__ldg(tsrc + (e0 + j))) << (8 * (j & 3));
+    }
+    const uint32_t crc_xor = p.crc_xor ? p.crc_xor[c] : 0u;
+    const uint64_t pad_begin = cd.payload_off + cd.len;
+    const uint64_t pad_end = cd.payload_off + align_up(cd.len, kPayloadAlign);
+    uint32_t h[16];
+    uint32_t pad = 0;  // OR of the padding bytes after the payload (< 256 of them)
+    if (mode_unpacks(MODE)) {
+      const uint4* src = reinterpret_cast<const uint4*>(p.packed + c * kHeaderBytes);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint4 v = src[q];
+        h[4 * q] = v.x;
+        h[4 * q + 1] = v.y;
+        h[4 * q + 2] = v.z;
+        h[4 * q + 3] = v.w;
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const uint64_t j = pad_begin + lane + 32u * q;
+        if (j < pad_end) pad |= p.packed[j];
+      }
+    }
+
+    // ---- 1. records: each shifted by the bytes after it in the chunk's body
+    // -- a multiplier the plan precomputed (1 for the last record, whose
+    // multiply is skipped), or (list mode, no-allocation entry) found here,
+    // last batch of 32 first so the byte count after each is known
     uint32_t raw = 0;
     double sq_rec = 0.0;
     uint32_t nf_rec = 0;
-    uint64_t carry = tail;
-    if (p.rec_mul && !p.ids) {
+    uint64_t carry = 0;
+    if (rec_mul) {
       uint32_t n = 0;
-      for (int64_t i = lane; i < n_recs; i += 32) {
+      if (lane < n_recs) {
+        raw = mul0 == kOne ? rec0.crc : gmul(rec0.crc, mul0);
+        n = rec0.nonfinite;
+      }
+      for (int64_t i = lane + 32; i < n_recs; i += 32) {
         const Record rec = p.recs[first_rec + i];
         raw ^= gmul(rec.crc, p.rec_mul[first_rec + i]);
         n += rec.nonfinite;
@@ -184,7 +260,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
       for (int m = 16; m >= 1; m >>= 1) n += __shfl_down_sync(kFull, n, m);
       nf_rec = __shfl_sync(kFull, n, 0);
     }
-    for (int64_t hi = (p.rec_mul && !p.ids) ? 0 : n_recs; hi > 0;) {
+    for (int64_t hi = rec_mul ? 0 : n_recs; hi > 0;) {
       const int64_t lo = hi > 32 ? hi - 32 : 0;
       const int64_t i = lo + lane;
       const bool have = i < hi;
@@ -208,22 +284,18 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
       nf_rec += __shfl_sync(kFull, n, 0);
       hi = lo;
     }
+    // the body's raw CRC, in every lane
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) raw ^= __shfl_xor_sync(kFull, raw, m);
     // the body's segment sums, in an order fixed by segment index alone
     if (values) {
       // pair-form slots are added as float pairs (TwoSum), tagged fp64 slots
       // (rare) in fp64, so the common case stays off the narrow fp64 pipe
-      const uint64_t n_seg = (body / kBlockBytes + kSegBlocks - 1) / kSegBlocks;
       float hi = 0.0f, lo = 0.0f;
       double dx = 0.0;
-      for (uint64_t k = lane; k < n_seg; k += 32) {
-        const double* slot = p.segs + cd.seg_base + k;
-        if (*reinterpret_cast<const uint64_t*>(slot) >> 63) {
-          dx += seg_value(slot);
-        } else {
-          const float2 f = *reinterpret_cast<const float2*>(slot);  // (lo, hi)
-          two_sum_pair(hi, lo, f.y, f.x);
-        }
-      }
+      if (lane < n_seg) add_slot(slot0, hi, lo, dx);
+      for (uint64_t k = lane + 32; k < n_seg; k += 32)
+        add_slot(reinterpret_cast<const uint64_t*>(p.segs + cd.seg_base)[k], hi, lo, dx);
 #pragma unroll
       for (int m = 16; m >= 1; m >>= 1) {
         const float oh = __shfl_down_sync(kFull, hi, m), ol = __shfl_down_sync(kFull, lo, m);
@@ -236,70 +308,66 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
       sq_rec = (static_cast<double>(hi) + static_cast<double>(lo)) + dx;
     }
 
-    // ---- 2. tail
-    const uint8_t* tsrc;
-    uint8_t* tdst = nullptr;
-    if (mode_unpacks(MODE)) {
-      tsrc = p.packed + cd.payload_off + body;
-      tdst = reinterpret_cast<uint8_t*>(cd.addr) + body;
-    } else {
-      tsrc = reinterpret_cast<const uint8_t*>(cd.addr) + body;
-      if (MODE == kModePack) tdst = p.packed + cd.payload_off + body;
-    }
-    // lane l takes the 16-byte piece that ends 16 * (31 - l) bytes before the
-    // tail's end (bytes before the tail are skipped: zero bytes leave a raw
-    // CRC run from zero unchanged), so its shift is a constant
+    // ---- 2. tail: copied, its elements summed, CRC'd a word at a time
+    // continuing from the body's raw CRC: a run started from state r equals
+    // one started from zero with r XORed into its first four bytes, so when
+    // the tail's first word is a whole word of one lane's piece (tail length
+    // a multiple of 4: always for fp32) that lane folds the body in there and
+    // the joined tail pieces give raw(body || tail) with no shift of the body;
+    // other tails (byte tensors, bf16) shift the body by x^(8 tail)
     float th = 0.0f, tl = 0.0f;  // the tail's sum of squares, as a float pair
     double tdx = 0.0;            // and its rare fp64 part
     uint32_t nf_tail = 0;
-    uint32_t tail_raw = 0;
-    const int32_t e1 = static_cast<int32_t>(tail) - 16 * (31 - static_cast<int32_t>(lane));
-    if (e1 > 0) {
-      const uint32_t b1 = static_cast<uint32_t>(e1);
-      const uint32_t b0 = b1 > 16u ? b1 - 16u : 0u;
-      uint32_t r = 0, word = 0;
-      for (uint32_t j = b0; j < b1; ++j) {
-        const uint32_t v = __ldg(tsrc + j);
-        r = crc_byte(T, r, v);
-        if (tdst) tdst[j] = static_cast<uint8_t>(v);
-        word |= v << (8 * (j & 3u));
+    if (tail != 0) {
+      uint32_t tail_raw = 0;
+      if (e0 + 16 > 0) {
+        if (tdst) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (e0 + j >= 0) tdst[e0 + j] = static_cast<uint8_t>(w[j >> 2] >> (8 * (j & 3)));
+        }
         if (values) {
-          if (cd.dtype == kDtF32 && (j & 3u) == 3u) {
-            tail_elem(kDtF32, word, nf_tail, th, tl, tdx);
-            word = 0;
-          } else if (cd.dtype == kDtBf16 && (j & 1u) == 1u) {
-            tail_elem(kDtBf16, (word >> (8 * ((j - 1) & 3u))) & 0xFFFFu, nf_tail, th, tl, tdx);
-            if ((j & 3u) == 3u) word = 0;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            if (cd.dtype == kDtF32) {
+              tail_elem(kDtF32, w[q], nf_tail, th, tl, tdx);
+            } else {
+              tail_elem(kDtBf16, w[q] & 0xFFFFu, nf_tail, th, tl, tdx);
+              tail_elem(kDtBf16, w[q] >> 16, nf_tail, th, tl, tdx);
+            }
           }
         }
+        if (e0 <= 0) {  // the tail's first byte is in this lane's piece
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (4 * q == -e0) w[q] ^= raw;  // only when it starts a word
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) tail_raw = mul_x32k(0, tail_raw ^ w[q]);
       }
-      tail_raw = r;
-    }
-    // lane l's piece ends 16 * (31 - l) bytes before the tail's end: join the
-    // 32 pieces in lane order; lane 0 holds the tail's raw CRC
-    tail_raw = join_lanes(tail_raw, 2, 5);
-    if (lane == 0) raw ^= tail_raw;
+      // lane l's piece ends 16 * (31 - l) bytes before the tail's end: join
+      // the 32 pieces in lane order into lane 0
+      const uint32_t joined = __shfl_sync(kFull, join_lanes(tail_raw, 2, 5), 0);
+      raw = (tail & 3u) == 0 ? joined : (shift_bytes(raw, tail) ^ joined);
 #pragma unroll
-    for (int m = 16; m >= 1; m >>= 1) {
-      raw ^= __shfl_xor_sync(kFull, raw, m);
-      nf_tail += __shfl_down_sync(kFull, nf_tail, m);
-      const float oh = __shfl_down_sync(kFull, th, m), ol = __shfl_down_sync(kFull, tl, m);
-      two_sum_pair(th, tl, oh, ol);
-    }
-    if (__any_sync(kFull, tdx != 0.0)) {
+      for (int m = 16; m >= 1; m >>= 1) {
+        nf_tail += __shfl_down_sync(kFull, nf_tail, m);
+        const float oh = __shfl_down_sync(kFull, th, m), ol = __shfl_down_sync(kFull, tl, m);
+        two_sum_pair(th, tl, oh, ol);
+      }
+      if (__any_sync(kFull, tdx != 0.0)) {
 #pragma unroll
-      for (int m = 16; m >= 1; m >>= 1) tdx += __shfl_down_sync(kFull, tdx, m);
+        for (int m = 16; m >= 1; m >>= 1) tdx += __shfl_down_sync(kFull, tdx, m);
+      }
     }
     const double sq_tail = (static_cast<double>(th) + static_cast<double>(tl)) + tdx;
 
     // ---- 3. preset and final XOR
-    const uint32_t crc = raw ^ (p.crc_xor ? p.crc_xor[c] : (shift_bytes(0xFFFFFFFFu, cd.len) ^ 0xFFFFFFFFu));
+    const uint32_t crc = raw ^ (p.crc_xor ? crc_xor : (shift_bytes(0xFFFFFFFFu, cd.len) ^ 0xFFFFFFFFu));
     // lane 0 holds the fixed-order sums and counts: every lane gets them
     const double sumsq = __shfl_sync(kFull, sq_rec + sq_tail, 0);
     const uint32_t nonfinite = __shfl_sync(kFull, nf_rec + nf_tail, 0);
 
-    const uint64_t pad_begin = cd.payload_off + cd.len;
-    const uint64_t pad_end = cd.payload_off + align_up(cd.len, kPayloadAlign);
     const uint64_t table_end = p.n_chunks * kHeaderBytes;
     const uint64_t gap_end = align_up(table_end, kPayloadAlign);
     const bool last = (c + 1 == p.n_chunks);
@@ -345,16 +413,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
         for (uint64_t j = table_end + lane * 16u; j < gap_end; j += 512)
           *reinterpret_cast<uint4*>(p.packed + j) = make_uint4(0, 0, 0, 0);
     } else if (mode_unpacks(MODE)) {  // unpack + verify
-      // every lane reads the (same) header and checks it against the plan
-      const uint4* src = reinterpret_cast<const uint4*>(p.packed + c * kHeaderBytes);
-      uint32_t h[16];
-      for (int q = 0; q < 4; ++q) {
-        const uint4 v = src[q];
-        h[4 * q] = v.x;
-        h[4 * q + 1] = v.y;
-        h[4 * q + 2] = v.z;
-        h[4 * q + 3] = v.w;
-      }
+      // every lane read the (same) header; check it against the plan
       const uint32_t hcrc = header_crc(T, h, lane);
       bool bad = (h[15] != hcrc) || h[0] != kMagic || (h[1] & 0xFFFFu) != kVersion || (h[1] >> 16) != cd.dtype ||
                  h[2] != static_cast<uint32_t>(c) || h[3] != static_cast<uint32_t>(c >> 32) ||
@@ -362,8 +421,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalizeParams p)
                  h[7] != static_cast<uint32_t>(cd.tensor_off >> 32) || h[8] != static_cast<uint32_t>(cd.len) ||
                  h[9] != static_cast<uint32_t>(cd.len >> 32) || h[10] != static_cast<uint32_t>(cd.payload_off) ||
                  h[11] != static_cast<uint32_t>(cd.payload_off >> 32) || h[5] != crc;
-      for (uint64_t j = pad_begin + lane; j < pad_end; j += 32)
-        if (p.packed[j] != 0) bad = true;
+      if (pad != 0) bad = true;
       if (last)
         for (uint64_t j = table_end + lane; j < gap_end; j += 32)
           if (p.packed[j] != 0) bad = true;

@@ -33,7 +33,7 @@ struct FinalizeParams {
   const Record* recs;
   const double* segs;
   const uint64_t* rec_nblk;
-  const uint32_t* rec_mul;  // per record: x^(8 * bytes after it in its chunk); null: computed here
+  const uint32_t* rec_mul;  // per record: x^(8 * bytes after it in its chunk's body); null: computed here
   const uint32_t* crc_xor;  // per chunk: CRC preset/final-XOR term for its length; null: computed here
   uint64_t n_chunks;        // chunks of the whole plan
   uint64_t c_begin, c_end;  // chunks to finalize: [c_begin, c_end), or list positions if ids != null
