@@ -62,6 +62,26 @@ def test_adversarial_sizes_and_chunks(chunk):
     compare_full(odd_tensors(1), chunk)
 
 
+@pytest.mark.parametrize("dt,esz", [(torch.uint8, 1), (torch.bfloat16, 2), (torch.float32, 4)])
+def test_every_tail_length(dt, esz):
+    """Chunk tails (len % 512) of every length up to 64 bytes and near 512, on
+    bodies of 0, 1 and several blocks, split over several warps: the body's
+    CRC is folded into a word-aligned tail, shifted past any other, and
+    absent when there is no tail."""
+    g = torch.Generator(device="cuda")
+    g.manual_seed(17)
+    tails = [t for t in list(range(0, 65)) + [500, 508, 510, 511] if t % esz == 0]
+    ts = []
+    for i, t in enumerate(tails):
+        nbytes = 512 * (0, 1, 7)[i % 3] + t
+        if dt == torch.uint8:
+            ts.append(torch.randint(0, 256, (nbytes,), generator=g, device="cuda", dtype=torch.uint8))
+        else:
+            ts.append(torch.randn(nbytes // esz, generator=g, device="cuda").to(dt))
+    compare_full(ts, 4096)  # one chunk per tensor
+    compare_full(ts, 1024)  # several chunks, tails only in the last
+
+
 @pytest.mark.parametrize("offset", [4, 8, 2])
 def test_misaligned_views(offset):
     ts = odd_tensors(2, offset)
