@@ -256,7 +256,9 @@ def run_flashrec(args):
             return int(nmis.item()), int(ndiv.item())
         return None
 
-    launches_per_step = (n_cls + 1) * 2 + (n_cls + 1) + (n_cls + 2) + 1  # sweeps + finalize + compaction + diff
+    # fingerprint: one sweep launch for all classes + finalize (twice); pack and
+    # unpack: one sweep launch per class + finalize (+ compaction); diff
+    launches_per_step = (min(n_cls, 1) + 1) * 2 + (n_cls + 1) + (n_cls + 2) + 1
 
     # correctness of the timed configuration: the injected flips are found
     for _ in range(args.warmup):

@@ -28,10 +28,28 @@
 
 using namespace frk;
 
+// Fingerprint sweeps launch every class of a batch in one kernel, sharing the
+// warps among the classes in proportion to their blocks weighted per element
+// type (percent of an fp32 block's cost).  A bf16 block costs a warp about a
+// quarter more than an fp32 block (twice the elements to square and add), so
+// the weight that lets both classes' warps finish together is about 125; the
+// weight matters (100 or 150 leave one class's warps finishing last).
+#ifndef FR_MIX_FP
+#define FR_MIX_FP 1
+#endif
+#ifndef FR_MIX_W_BF16
+#define FR_MIX_W_BF16 125
+#endif
+#ifndef FR_MIX_W_BYTES
+#define FR_MIX_W_BYTES 100
+#endif
+
+
 namespace {
 
 // One sweep class of one batch: its kernel specialization and its slices of
-// the decomposition's warp and chunk-list tables.
+// the decomposition's warp and chunk-list tables (a mixed decomposition has
+// one entry per batch covering all its classes).
 struct SweepClass {
   uint32_t dtype = 0;
   bool aligned = false;
@@ -47,6 +65,7 @@ struct BatchInfo {
 // Per-warp work of every batch, with the chunk table that carries this
 // decomposition's block offsets and record ranges.
 struct Decomp {
+  bool mixed = false;  // one launch per batch for all its classes
   int n_ctas = 0;
   uint32_t n_warps = 0;  // per class launch: n_ctas * warps per CTA
   std::vector<BatchInfo> batches;
@@ -177,10 +196,13 @@ void free_device(fr_plan p) {
 // overlap gets one record.  Records are numbered batch by batch, class
 // by class, so each chunk's records are consecutive.  `min_recs`: record slots
 // to allocate at least (list-mode calls use one slot per listed chunk).
+// Plain: every class gets all n_ctas * warps_per_cta warps (one launch per
+// class).  Mixed: the classes of a batch share them in proportion to their
+// weighted blocks, each class's warps spread round-robin over the CTAs.
 cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<uint64_t>& bounds, int n_ctas,
-                         int warps_per_cta,
-                         uint64_t min_recs, Decomp& D) {
+                         int warps_per_cta, bool mixed, uint64_t min_recs, Decomp& D) {
   const uint64_t W = static_cast<uint64_t>(n_ctas) * warps_per_cta;
+  D.mixed = mixed;
   D.n_ctas = n_ctas;
   D.n_warps = static_cast<uint32_t>(W);
   std::vector<ChunkDesc> chunks = base;
@@ -203,36 +225,109 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
       d.blk_begin = class_blocks[d.sweep_class];
       class_blocks[d.sweep_class] += d.len / kBlockBytes;
     }
+    // the batch's classes: chunk lists and, per class, the class-stream block
+    // where each segment starts (warp ranges start on segment boundaries)
+    struct Cls {
+      uint32_t cls;
+      uint64_t list_off;
+      std::vector<uint64_t> seg_start;
+    };
+    std::vector<Cls> cl;
     for (uint32_t cls = 0; cls < 6; ++cls) {
-      const uint64_t blk = class_blocks[cls];
-      if (blk == 0) continue;
+      if (class_blocks[cls] == 0) continue;
+      Cls q;
+      q.cls = cls;
+      q.list_off = lists.size();
+      for (uint64_t c = bi.c_begin; c < bi.c_end; ++c)
+        if (chunks[c].sweep_class == cls && chunks[c].len >= static_cast<uint64_t>(kBlockBytes))
+          lists.push_back(static_cast<uint32_t>(c));
+      for (size_t i = q.list_off; i < lists.size(); ++i) {
+        const ChunkDesc& d = chunks[lists[i]];
+        for (uint64_t j = 0; j < d.len / kBlockBytes; j += kSegBlocks) q.seg_start.push_back(d.blk_begin + j);
+      }
+      q.seg_start.push_back(class_blocks[cls]);
+      cl.push_back(std::move(q));
+    }
+    if (cl.empty()) {
+      D.batches.push_back(bi);
+      continue;
+    }
+    // warps per class, and (mixed) the batch-warp slot of each class's j-th warp
+    std::vector<uint64_t> wc(cl.size(), W);
+    std::vector<std::vector<uint64_t>> slot(cl.size());
+    const uint64_t warp_base = warps.size();
+    if (mixed) {
+      std::vector<double> cost(cl.size());
+      double total = 0.0;
+      for (size_t q = 0; q < cl.size(); ++q) {
+        const uint32_t dt = cl[q].cls / 2;
+        const double w = dt == kDtF32 ? 100.0 : (dt == kDtBf16 ? FR_MIX_W_BF16 : FR_MIX_W_BYTES);
+        cost[q] = static_cast<double>(class_blocks[cl[q].cls]) * w;
+        total += cost[q];
+      }
+      uint64_t given = 0;
+      for (size_t q = 0; q < cl.size(); ++q) {
+        wc[q] = std::max<uint64_t>(1, static_cast<uint64_t>(static_cast<double>(W) * cost[q] / total));
+        given += wc[q];
+      }
+      while (given < W) {  // the rest to the class furthest below its share
+        size_t best = 0;
+        double gap = -1e300;
+        for (size_t q = 0; q < cl.size(); ++q) {
+          const double g = static_cast<double>(W) * cost[q] / total - static_cast<double>(wc[q]);
+          if (g > gap) gap = g, best = q;
+        }
+        ++wc[best];
+        ++given;
+      }
+      while (given > W) {  // (only when many tiny classes each took one)
+        size_t best = 0;
+        for (size_t q = 1; q < cl.size(); ++q)
+          if (wc[q] > wc[best]) best = q;
+        --wc[best];
+        --given;
+      }
+      // slot i is warp i / n_ctas of CTA i % n_ctas; each slot goes to the
+      // class furthest behind its share of the slots so far
+      std::vector<uint64_t> done(cl.size(), 0);
+      for (uint64_t i = 0; i < W; ++i) {
+        size_t best = cl.size();
+        double gap = -1e300;
+        for (size_t q = 0; q < cl.size(); ++q) {
+          if (done[q] == wc[q]) continue;
+          const double g = static_cast<double>(wc[q]) * static_cast<double>(i + 1) / static_cast<double>(W) -
+                           static_cast<double>(done[q]);
+          if (g > gap) gap = g, best = q;
+        }
+        slot[best].push_back((i % n_ctas) * warps_per_cta + i / n_ctas);
+        ++done[best];
+      }
+      warps.resize(warp_base + W);
+      SweepClass sc;
+      sc.warp_off = warp_base;
+      sc.list_off = 0;
+      bi.classes.push_back(sc);
+    }
+    for (size_t q = 0; q < cl.size(); ++q) {
+      const uint32_t cls = cl[q].cls;
+      const size_t lbase = cl[q].list_off;
+      const std::vector<uint64_t>& seg_start = cl[q].seg_start;
+      const uint64_t n_seg = seg_start.size() - 1, Wq = wc[q];
       SweepClass sc;
       sc.dtype = cls / 2;
       sc.aligned = (cls & 1u) != 0;
       sc.warp_off = warps.size();
-      sc.list_off = lists.size();
-      for (uint64_t c = bi.c_begin; c < bi.c_end; ++c)
-        if (chunks[c].sweep_class == cls && chunks[c].len >= static_cast<uint64_t>(kBlockBytes))
-          lists.push_back(static_cast<uint32_t>(c));
-      const size_t lbase = sc.list_off;
-      // warp ranges start on segment boundaries: cut the class's segments
-      // (not its blocks) evenly, then convert to block ranges
-      std::vector<uint64_t> seg_start;  // class-stream block where each segment starts
-      for (size_t q = lbase; q < lists.size(); ++q) {
-        const ChunkDesc& d = chunks[lists[q]];
-        const uint64_t nb = d.len / kBlockBytes;
-        for (uint64_t j = 0; j < nb; j += kSegBlocks) seg_start.push_back(d.blk_begin + j);
-      }
-      const uint64_t n_seg = seg_start.size();
-      seg_start.push_back(blk);
+      sc.list_off = lbase;
       uint64_t k = 0;  // walks the class list monotonically
-      for (uint64_t w = 0; w < W; ++w) {
-        const uint64_t b0 = seg_start[n_seg * w / W], b1 = seg_start[n_seg * (w + 1) / W];
+      for (uint64_t w = 0; w < Wq; ++w) {
+        const uint64_t b0 = seg_start[n_seg * w / Wq], b1 = seg_start[n_seg * (w + 1) / Wq];
         WarpDesc wd;
         std::memset(&wd, 0, sizeof wd);
         wd.blk_begin = b0;
         wd.nblk = b1 - b0;
         wd.rec_base = static_cast<uint32_t>(rec_nblk.size());
+        wd.cls = cls;
+        wd.list_off = static_cast<uint32_t>(lbase);
         if (b1 > b0) {
           while (b0 >= chunks[lists[lbase + k]].blk_begin + chunks[lists[lbase + k]].len / kBlockBytes) ++k;
           wd.first_chunk = static_cast<uint32_t>(k);
@@ -249,9 +344,12 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
             if (bb == end) ++j;
           }
         }
-        warps.push_back(wd);
+        if (mixed)
+          warps[warp_base + slot[q][w]] = wd;
+        else
+          warps.push_back(wd);
       }
-      bi.classes.push_back(sc);
+      if (!mixed) bi.classes.push_back(sc);
     }
     D.batches.push_back(bi);
   }
@@ -280,7 +378,9 @@ fr_status run_batches(fr_plan p, const Decomp& D, int mode, uint8_t* packed, FpE
       sp.packed = packed;
       sp.n_warps = D.n_warps;
       cudaError_t e;
-      if (mode == kModeFingerprint)
+      if (D.mixed)  // (fingerprint decompositions only)
+        e = launch_sweep_fp_mixed(sp, D.n_ctas, s);
+      else if (mode == kModeFingerprint)
         e = launch_sweep_fp(sc.dtype, sc.aligned, sp, D.n_ctas, s);
       else if (mode == kModePack)
         e = launch_sweep_pack(sc.dtype, sc.aligned, sp, D.n_ctas, s);
@@ -500,9 +600,11 @@ fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, u
   // ---- decompositions
   e = cudaSuccess;
   if (n_chunks > 0) {
-    std::vector<int> counts;  // distinct warps-per-CTA counts of the modes
+    // distinct decompositions of the modes: warps per CTA, and whether mixed
+    // (the fingerprint's, so the fingerprint is always geo 0)
+    std::vector<int> counts;  // 2 * warps + mixed
     for (int m = 0; m < 4; ++m) {
-      const int w = sweep_warps(m);
+      const int w = 2 * sweep_warps(m) + ((m == kModeFingerprint && FR_MIX_FP) ? 1 : 0);
       int g = 0;
       while (g < static_cast<int>(counts.size()) && counts[g] != w) ++g;
       if (g == static_cast<int>(counts.size())) counts.push_back(w);
@@ -511,7 +613,8 @@ fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, u
     p->whole.resize(counts.size());
     p->batched.resize(counts.size());
     for (size_t g = 0; e == cudaSuccess && g < counts.size(); ++g)
-      e = build_decomp(p->chunks, {0, n_chunks}, n_sm, counts[g], g == 0 ? n_chunks : 0, p->whole[g]);
+      e = build_decomp(p->chunks, {0, n_chunks}, n_sm, counts[g] / 2, (counts[g] & 1) != 0, g == 0 ? n_chunks : 0,
+                       p->whole[g]);
     if (e == cudaSuccess && p->n_batches > 1) {
       // batch starts at about equal state bytes, every batch non-empty
       std::vector<uint64_t> bounds(1, 0);
@@ -526,7 +629,8 @@ fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, u
       for (size_t i = 1; i < bounds.size(); ++i)
         if (bounds[i] <= bounds[i - 1]) bounds[i] = bounds[i - 1] + 1;
       for (size_t g = 0; e == cudaSuccess && g < counts.size(); ++g)
-        e = build_decomp(p->chunks, bounds, std::max(1, n_sm / 2), counts[g], 0, p->batched[g]);
+        e = build_decomp(p->chunks, bounds, std::max(1, n_sm / 2), counts[g] / 2, (counts[g] & 1) != 0, 0,
+                         p->batched[g]);
     }
   }
   if (e == cudaSuccess && p->n_segs) e = cudaMalloc(&p->d_segs, p->n_segs * sizeof(double));

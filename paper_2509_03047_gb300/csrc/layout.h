@@ -72,7 +72,8 @@ struct WarpDesc {        // 32 bytes
   uint64_t nblk;         // blocks in the range (0: idle warp)
   uint32_t first_chunk;  // position, in the class's chunk list, of the chunk holding blk_begin
   uint32_t rec_base;     // record index of the first piece
-  uint64_t pad;
+  uint32_t cls;          // mixed launches: the sweep class of the warp's chunks
+  uint32_t list_off;     // mixed launches: where that class's chunk list starts
 };
 static_assert(sizeof(WarpDesc) == 32, "WarpDesc layout");
 

@@ -3,10 +3,17 @@
 
 namespace frk {
 
-cudaError_t configure_sweep_fp() { return configure_mode<kModeFingerprint>(); }
+cudaError_t configure_sweep_fp() {
+  const cudaError_t e = configure_mode<kModeFingerprint>();
+  return e == cudaSuccess ? configure_mixed<kModeFingerprint>() : e;
+}
 
 cudaError_t launch_sweep_fp(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s) {
   return launch_mode<kModeFingerprint>(dtype, aligned, p, n_ctas, s);
+}
+
+cudaError_t launch_sweep_fp_mixed(const SweepParams& p, int n_ctas, cudaStream_t s) {
+  return launch_mixed<kModeFingerprint>(p, n_ctas, s);
 }
 
 }  // namespace frk

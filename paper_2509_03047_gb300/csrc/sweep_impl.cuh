@@ -550,21 +550,17 @@ __device__ __forceinline__ void sweep_piece_al(const uint8_t* tensor, uint8_t* p
     sweep_piece<MODE, DT, AL, 16>(tensor, packed, n, lane, rec, segs);
 }
 
-// One kernel per (mode, element type, alignment class).  ALIGNED: every
-// tensor of the class is 16-byte aligned (128-bit loads and stores); else the
-// tensor side uses 32-bit or byte accesses, chosen per piece.
+// One warp's range of its class's block stream: the pieces it overlaps, in
+// order.  ALIGNED: every tensor of the class is 16-byte aligned (128-bit
+// loads and stores); else the tensor side uses 32-bit or byte accesses, chosen
+// per piece.
 template <int MODE, int DT, bool ALIGNED>
-__global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_kernel(SweepParams p) {
-  fill_tables();
-  __syncthreads();
-  const uint32_t lane = threadIdx.x & 31u;
-  const uint32_t w = blockIdx.x * Cta<MODE>::kWarps + (threadIdx.x >> 5);
-  if (w >= p.n_warps) return;
-  const WarpDesc wd = p.warps[w];
+__device__ __forceinline__ void sweep_warp(const SweepParams& p, const WarpDesc& wd, const uint32_t* class_chunks,
+                                           uint32_t lane) {
   uint64_t b = wd.blk_begin, left = wd.nblk;
   uint32_t k = wd.first_chunk, r = wd.rec_base;
   while (left > 0) {
-    const ChunkDesc cd = p.chunks[p.class_chunks[k]];
+    const ChunkDesc cd = p.chunks[class_chunks[k]];
     const uint64_t nb = cd.len / kBlockBytes;
     const uint64_t off = b - cd.blk_begin;
     const uint64_t n = (left < nb - off) ? left : nb - off;
@@ -582,6 +578,40 @@ __global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_kernel(SweepPara
     b += n;
     left -= n;
     ++k;
+  }
+}
+
+// One kernel per (mode, element type, alignment class).
+template <int MODE, int DT, bool ALIGNED>
+__global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_kernel(SweepParams p) {
+  fill_tables();
+  __syncthreads();
+  const uint32_t lane = threadIdx.x & 31u;
+  const uint32_t w = blockIdx.x * Cta<MODE>::kWarps + (threadIdx.x >> 5);
+  if (w >= p.n_warps) return;
+  sweep_warp<MODE, DT, ALIGNED>(p, p.warps[w], p.class_chunks, lane);
+}
+
+// Every class of a batch in one launch: each warp sweeps a range of its own
+// class (wd.cls, chunk list at class_chunks + wd.list_off), and the plan
+// spreads each class's warps over all CTAs, so warps that wait on memory and
+// warps that are bound by instruction issue share every SM.
+template <int MODE>
+__global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_mixed_kernel(SweepParams p) {
+  fill_tables();
+  __syncthreads();
+  const uint32_t lane = threadIdx.x & 31u;
+  const uint32_t w = blockIdx.x * Cta<MODE>::kWarps + (threadIdx.x >> 5);
+  if (w >= p.n_warps) return;
+  const WarpDesc wd = p.warps[w];
+  const uint32_t* list = p.class_chunks + wd.list_off;
+  switch (wd.cls) {
+    case kDtF32 * 2 + 1: sweep_warp<MODE, kDtF32, true>(p, wd, list, lane); break;
+    case kDtBf16 * 2 + 1: sweep_warp<MODE, kDtBf16, true>(p, wd, list, lane); break;
+    case kDtBytes * 2 + 1: sweep_warp<MODE, kDtBytes, true>(p, wd, list, lane); break;
+    case kDtF32 * 2: sweep_warp<MODE, kDtF32, false>(p, wd, list, lane); break;
+    case kDtBf16 * 2: sweep_warp<MODE, kDtBf16, false>(p, wd, list, lane); break;
+    default: sweep_warp<MODE, kDtBytes, false>(p, wd, list, lane); break;
   }
 }
 
@@ -663,6 +693,17 @@ cudaError_t configure_mode() {
     if (e == cudaSuccess) e = configure_one<MODE, kDtF32, false>();
   }
   return e;
+}
+
+template <int MODE>
+cudaError_t configure_mixed() {
+  return cudaFuncSetAttribute(sweep_mixed_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTableBytes);
+}
+
+template <int MODE>
+cudaError_t launch_mixed(const SweepParams& p, int n_ctas, cudaStream_t s) {
+  sweep_mixed_kernel<MODE><<<n_ctas, Cta<MODE>::kThreads, kTableBytes, s>>>(p);
+  return cudaGetLastError();
 }
 
 template <int MODE>
