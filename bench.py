@@ -256,9 +256,10 @@ def run_flashrec(args):
             return int(nmis.item()), int(ndiv.item())
         return None
 
-    # fingerprint: one sweep launch for all classes + finalize (twice); pack and
-    # unpack: one sweep launch per class + finalize (+ compaction); diff
-    launches_per_step = (min(n_cls, 1) + 1) * 2 + (n_cls + 1) + (n_cls + 2) + 1
+    # every call: one sweep launch for all classes + finalize; fingerprint
+    # twice, unpack with its compaction; diff
+    sweeps = min(n_cls, 1)
+    launches_per_step = (sweeps + 1) * 2 + (sweeps + 1) + (sweeps + 2) + 1
 
     # correctness of the timed configuration: the injected flips are found
     for _ in range(args.warmup):

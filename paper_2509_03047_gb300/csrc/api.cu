@@ -43,6 +43,14 @@ using namespace frk;
 #ifndef FR_MIX_W_BYTES
 #define FR_MIX_W_BYTES 100
 #endif
+// Pack and unpack likewise (memory-bound in every class: equal weights); one
+// launch per call instead of one per class saves a launch and a ramp.
+#ifndef FR_MIX_PACK
+#define FR_MIX_PACK 1
+#endif
+#ifndef FR_MIX_W_BF16_PACK
+#define FR_MIX_W_BF16_PACK 100
+#endif
 
 
 namespace {
@@ -200,7 +208,8 @@ void free_device(fr_plan p) {
 // class).  Mixed: the classes of a batch share them in proportion to their
 // weighted blocks, each class's warps spread round-robin over the CTAs.
 cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<uint64_t>& bounds, int n_ctas,
-                         int warps_per_cta, bool mixed, uint64_t min_recs, Decomp& D) {
+                         int warps_per_cta, int mix, uint64_t min_recs, Decomp& D) {
+  const bool mixed = mix != 0;  // 1: fingerprint weights, 2: pack / unpack weights
   const uint64_t W = static_cast<uint64_t>(n_ctas) * warps_per_cta;
   D.mixed = mixed;
   D.n_ctas = n_ctas;
@@ -261,7 +270,8 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
       double total = 0.0;
       for (size_t q = 0; q < cl.size(); ++q) {
         const uint32_t dt = cl[q].cls / 2;
-        const double w = dt == kDtF32 ? 100.0 : (dt == kDtBf16 ? FR_MIX_W_BF16 : FR_MIX_W_BYTES);
+        const double w_bf16 = mix == 1 ? FR_MIX_W_BF16 : FR_MIX_W_BF16_PACK;
+        const double w = dt == kDtF32 ? 100.0 : (dt == kDtBf16 ? w_bf16 : FR_MIX_W_BYTES);
         cost[q] = static_cast<double>(class_blocks[cl[q].cls]) * w;
         total += cost[q];
       }
@@ -378,8 +388,11 @@ fr_status run_batches(fr_plan p, const Decomp& D, int mode, uint8_t* packed, FpE
       sp.packed = packed;
       sp.n_warps = D.n_warps;
       cudaError_t e;
-      if (D.mixed)  // (fingerprint decompositions only)
-        e = launch_sweep_fp_mixed(sp, D.n_ctas, s);
+      if (D.mixed)
+        e = mode == kModeFingerprint ? launch_sweep_fp_mixed(sp, D.n_ctas, s)
+            : mode == kModePack      ? launch_sweep_pack_mixed(sp, D.n_ctas, s)
+            : mode == kModeUnpackFp  ? launch_sweep_unpack_fp_mixed(sp, D.n_ctas, s)
+                                     : launch_sweep_unpack_mixed(sp, D.n_ctas, s);
       else if (mode == kModeFingerprint)
         e = launch_sweep_fp(sc.dtype, sc.aligned, sp, D.n_ctas, s);
       else if (mode == kModePack)
@@ -600,11 +613,12 @@ fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, u
   // ---- decompositions
   e = cudaSuccess;
   if (n_chunks > 0) {
-    // distinct decompositions of the modes: warps per CTA, and whether mixed
-    // (the fingerprint's, so the fingerprint is always geo 0)
-    std::vector<int> counts;  // 2 * warps + mixed
+    // distinct decompositions of the modes: warps per CTA and mixing (none,
+    // with the fingerprint's weights, with pack's); the fingerprint's is geo 0
+    std::vector<int> counts;  // 3 * warps + mix
     for (int m = 0; m < 4; ++m) {
-      const int w = 2 * sweep_warps(m) + ((m == kModeFingerprint && FR_MIX_FP) ? 1 : 0);
+      const int mix = m == kModeFingerprint ? (FR_MIX_FP ? 1 : 0) : (FR_MIX_PACK ? 2 : 0);
+      const int w = 3 * sweep_warps(m) + mix;
       int g = 0;
       while (g < static_cast<int>(counts.size()) && counts[g] != w) ++g;
       if (g == static_cast<int>(counts.size())) counts.push_back(w);
@@ -613,8 +627,7 @@ fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, u
     p->whole.resize(counts.size());
     p->batched.resize(counts.size());
     for (size_t g = 0; e == cudaSuccess && g < counts.size(); ++g)
-      e = build_decomp(p->chunks, {0, n_chunks}, n_sm, counts[g] / 2, (counts[g] & 1) != 0, g == 0 ? n_chunks : 0,
-                       p->whole[g]);
+      e = build_decomp(p->chunks, {0, n_chunks}, n_sm, counts[g] / 3, counts[g] % 3, g == 0 ? n_chunks : 0, p->whole[g]);
     if (e == cudaSuccess && p->n_batches > 1) {
       // batch starts at about equal state bytes, every batch non-empty
       std::vector<uint64_t> bounds(1, 0);
@@ -629,8 +642,7 @@ fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, u
       for (size_t i = 1; i < bounds.size(); ++i)
         if (bounds[i] <= bounds[i - 1]) bounds[i] = bounds[i - 1] + 1;
       for (size_t g = 0; e == cudaSuccess && g < counts.size(); ++g)
-        e = build_decomp(p->chunks, bounds, std::max(1, n_sm / 2), counts[g] / 2, (counts[g] & 1) != 0, 0,
-                         p->batched[g]);
+        e = build_decomp(p->chunks, bounds, std::max(1, n_sm / 2), counts[g] / 3, counts[g] % 3, 0, p->batched[g]);
     }
   }
   if (e == cudaSuccess && p->n_segs) e = cudaMalloc(&p->d_segs, p->n_segs * sizeof(double));

@@ -88,6 +88,9 @@ cudaError_t launch_sweep_fp(uint32_t dtype, bool aligned, const SweepParams& p, 
 // Every class of a batch in one fingerprint launch (per-warp class in WarpDesc;
 // class_chunks = the whole chunk-list table).
 cudaError_t launch_sweep_fp_mixed(const SweepParams& p, int n_ctas, cudaStream_t s);
+cudaError_t launch_sweep_pack_mixed(const SweepParams& p, int n_ctas, cudaStream_t s);
+cudaError_t launch_sweep_unpack_mixed(const SweepParams& p, int n_ctas, cudaStream_t s);
+cudaError_t launch_sweep_unpack_fp_mixed(const SweepParams& p, int n_ctas, cudaStream_t s);
 cudaError_t launch_sweep_pack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
 cudaError_t launch_sweep_unpack(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s);
 cudaError_t launch_list_pack(const ListParams& p, cudaStream_t s);

@@ -605,6 +605,13 @@ __global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_mixed_kernel(Swe
   if (w >= p.n_warps) return;
   const WarpDesc wd = p.warps[w];
   const uint32_t* list = p.class_chunks + wd.list_off;
+  if constexpr (!mode_sums(MODE)) {  // (copies and checksums bytes only: no element types)
+    if (wd.cls & 1u)
+      sweep_warp<MODE, kDtBytes, true>(p, wd, list, lane);
+    else
+      sweep_warp<MODE, kDtBytes, false>(p, wd, list, lane);
+    return;
+  }
   switch (wd.cls) {
     case kDtF32 * 2 + 1: sweep_warp<MODE, kDtF32, true>(p, wd, list, lane); break;
     case kDtBf16 * 2 + 1: sweep_warp<MODE, kDtBf16, true>(p, wd, list, lane); break;

@@ -5,10 +5,17 @@
 
 namespace frk {
 
-cudaError_t configure_sweep_unpack_fp() { return configure_mode<kModeUnpackFp>(); }
+cudaError_t configure_sweep_unpack_fp() {
+  const cudaError_t e = configure_mode<kModeUnpackFp>();
+  return e == cudaSuccess ? configure_mixed<kModeUnpackFp>() : e;
+}
 
 cudaError_t launch_sweep_unpack_fp(uint32_t dtype, bool aligned, const SweepParams& p, int n_ctas, cudaStream_t s) {
   return launch_mode<kModeUnpackFp>(dtype, aligned, p, n_ctas, s);
+}
+
+cudaError_t launch_sweep_unpack_fp_mixed(const SweepParams& p, int n_ctas, cudaStream_t s) {
+  return launch_mixed<kModeUnpackFp>(p, n_ctas, s);
 }
 
 cudaError_t launch_list_unpack_fp(const ListParams& p, cudaStream_t s) { return launch_list<kModeUnpackFp>(p, s); }
