@@ -18,7 +18,7 @@ OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libflashrec.so")
 SOURCES = ["sweep_fp.cu", "sweep_pack.cu", "sweep_unpack.cu", "sweep_unpack_fp.cu", "finalize.cu", "api.cu",
            "static_fingerprint.cu"]
-HEADERS = ["gf2.cuh", "layout.h", "kernels.h", "sweep_impl.cuh"]
+HEADERS = ["gf2.cuh", "layout.h", "kernels.h", "sweep_impl.cuh", "warp_share.h"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",

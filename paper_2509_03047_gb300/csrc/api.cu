@@ -25,31 +25,19 @@
 #include "gf2.cuh"
 #include "kernels.h"
 #include "layout.h"
+#include "warp_share.h"
 
 using namespace frk;
 
-// Fingerprint sweeps launch every class of a batch in one kernel, sharing the
-// warps among the classes in proportion to their blocks weighted per element
-// type (percent of an fp32 block's cost).  A bf16 block costs a warp about a
-// quarter more than an fp32 block (twice the elements to square and add), so
-// the weight that lets both classes' warps finish together is about 125; the
-// weight matters (100 or 150 leave one class's warps finishing last).
+// Each call launches one sweep kernel for every class of a batch, its warps
+// shared among the classes by weighted blocks (warp_share.h); the weight
+// matters for the fingerprint (a bf16 weight of 100 or 150 instead of 125
+// leaves one class's warps finishing last).  Off: one launch per class.
 #ifndef FR_MIX_FP
 #define FR_MIX_FP 1
 #endif
-#ifndef FR_MIX_W_BF16
-#define FR_MIX_W_BF16 125
-#endif
-#ifndef FR_MIX_W_BYTES
-#define FR_MIX_W_BYTES 100
-#endif
-// Pack and unpack likewise (memory-bound in every class: equal weights); one
-// launch per call instead of one per class saves a launch and a ramp.
 #ifndef FR_MIX_PACK
 #define FR_MIX_PACK 1
-#endif
-#ifndef FR_MIX_W_BF16_PACK
-#define FR_MIX_W_BF16_PACK 100
 #endif
 
 
@@ -266,52 +254,13 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
     std::vector<std::vector<uint64_t>> slot(cl.size());
     const uint64_t warp_base = warps.size();
     if (mixed) {
-      std::vector<double> cost(cl.size());
-      double total = 0.0;
-      for (size_t q = 0; q < cl.size(); ++q) {
-        const uint32_t dt = cl[q].cls / 2;
-        const double w_bf16 = mix == 1 ? FR_MIX_W_BF16 : FR_MIX_W_BF16_PACK;
-        const double w = dt == kDtF32 ? 100.0 : (dt == kDtBf16 ? w_bf16 : FR_MIX_W_BYTES);
-        cost[q] = static_cast<double>(class_blocks[cl[q].cls]) * w;
-        total += cost[q];
-      }
-      uint64_t given = 0;
-      for (size_t q = 0; q < cl.size(); ++q) {
-        wc[q] = std::max<uint64_t>(1, static_cast<uint64_t>(static_cast<double>(W) * cost[q] / total));
-        given += wc[q];
-      }
-      while (given < W) {  // the rest to the class furthest below its share
-        size_t best = 0;
-        double gap = -1e300;
-        for (size_t q = 0; q < cl.size(); ++q) {
-          const double g = static_cast<double>(W) * cost[q] / total - static_cast<double>(wc[q]);
-          if (g > gap) gap = g, best = q;
-        }
-        ++wc[best];
-        ++given;
-      }
-      while (given > W) {  // (only when many tiny classes each took one)
-        size_t best = 0;
-        for (size_t q = 1; q < cl.size(); ++q)
-          if (wc[q] > wc[best]) best = q;
-        --wc[best];
-        --given;
-      }
-      // slot i is warp i / n_ctas of CTA i % n_ctas; each slot goes to the
-      // class furthest behind its share of the slots so far
-      std::vector<uint64_t> done(cl.size(), 0);
-      for (uint64_t i = 0; i < W; ++i) {
-        size_t best = cl.size();
-        double gap = -1e300;
-        for (size_t q = 0; q < cl.size(); ++q) {
-          if (done[q] == wc[q]) continue;
-          const double g = static_cast<double>(wc[q]) * static_cast<double>(i + 1) / static_cast<double>(W) -
-                           static_cast<double>(done[q]);
-          if (g > gap) gap = g, best = q;
-        }
-        slot[best].push_back((i % n_ctas) * warps_per_cta + i / n_ctas);
-        ++done[best];
-      }
+      double cost[6];
+      for (size_t q = 0; q < cl.size(); ++q)
+        cost[q] = static_cast<double>(class_blocks[cl[q].cls]) * block_weight(cl[q].cls / 2, mix);
+      share_warps(cost, static_cast<int>(cl.size()), W, wc.data());
+      std::vector<uint32_t> slots(cl.size() * W);
+      spread_warps(wc.data(), static_cast<int>(cl.size()), W, n_ctas, warps_per_cta, slots.data(), W);
+      for (size_t q = 0; q < cl.size(); ++q) slot[q].assign(slots.begin() + q * W, slots.begin() + q * W + wc[q]);
       warps.resize(warp_base + W);
       SweepClass sc;
       sc.warp_off = warp_base;

@@ -30,6 +30,7 @@
 #include "gf2.cuh"
 #include "kernels.h"
 #include "layout.h"
+#include "warp_share.h"
 
 using namespace frk;
 
@@ -37,9 +38,8 @@ namespace {
 
 // Limits of the static variant.
 constexpr uint64_t kMaxChunks = FR_STATIC_MAX_CHUNKS;
-constexpr uint64_t kMaxWarpsPerClass = 160 * sweep_warps(kModeFingerprint);  // up to 160 SMs
+constexpr uint64_t kMaxWarps = 160 * sweep_warps(kModeFingerprint);  // up to 160 SMs, shared by the classes
 constexpr uint64_t kClasses = 6;
-constexpr uint64_t kMaxWarps = kClasses * kMaxWarpsPerClass;
 constexpr uint64_t kMaxRecs = kMaxWarps + kMaxChunks;
 constexpr uint64_t kMaxSegs = FR_STATIC_MAX_SEGMENTS;  // 16 KiB sum segments
 
@@ -65,6 +65,7 @@ struct HostTables {
   WarpDesc warps[kMaxWarps];
   uint64_t rec_nblk[kMaxRecs];
   uint64_t seg_start[kMaxSegs + 1];  // per class: block where each segment starts
+  uint32_t slot[kClasses * kMaxWarps];  // per class: launch-warp index of its j-th warp
 };
 HostTables g_host;
 std::mutex g_mu;
@@ -129,7 +130,7 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
   e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
   const uint64_t W = static_cast<uint64_t>(n_sm) * sweep_warps(kModeFingerprint);
-  if (W > kMaxWarpsPerClass) return fail(FR_ERR_INVALID_ARG, "GPU has more SMs than the static tables hold");
+  if (W > kMaxWarps) return fail(FR_ERR_INVALID_ARG, "GPU has more SMs than the static tables hold");
 
   std::lock_guard<std::mutex> lk(g_mu);
   uint8_t* scratch = nullptr;
@@ -161,37 +162,49 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
       class_blocks[cls] += d.len / kBlockBytes;
     }
   }
-  struct Launch {
-    uint32_t dtype;
-    bool aligned;
-    uint64_t warp_off, list_off;
-  } launches[kClasses];
-  int n_launch = 0;
-  uint64_t n_warps = 0, n_lists = 0, n_recs = 0;
+  // one launch for every class: the W warps shared by weighted blocks, each
+  // class's warps spread over the CTAs (warp_share.h)
+  uint32_t cls_of[kClasses];
+  double cost[kClasses];
+  uint64_t wc[kClasses];
+  int n_cls = 0;
   for (uint32_t cls = 0; cls < kClasses; ++cls) {
-    const uint64_t blk = class_blocks[cls];
-    if (blk == 0) continue;
-    Launch L{cls / 2, (cls & 1u) != 0, n_warps, n_lists};
+    if (class_blocks[cls] == 0) continue;
+    cls_of[n_cls] = cls;
+    cost[n_cls] = static_cast<double>(class_blocks[cls]) * block_weight(cls / 2, kShareFingerprint);
+    ++n_cls;
+  }
+  if (n_cls > 0) {
+    share_warps(cost, n_cls, W, wc);
+    spread_warps(wc, n_cls, W, n_sm, sweep_warps(kModeFingerprint), h.slot, kMaxWarps);
+  }
+  uint64_t n_lists = 0, n_recs = 0;
+  for (int q = 0; q < n_cls; ++q) {
+    const uint32_t cls = cls_of[q];
+    const uint64_t blk = class_blocks[cls], Wq = wc[q];
+    const uint64_t list_off = n_lists;
     for (uint64_t i = 0; i < n_chunks; ++i)
       if (h.chunks[i].sweep_class == cls && h.chunks[i].len >= static_cast<uint64_t>(kBlockBytes))
         h.lists[n_lists++] = static_cast<uint32_t>(i);
-    const uint32_t* list = h.lists + L.list_off;
+    const uint32_t* list = h.lists + list_off;
     // warp ranges start on 16 KiB segment boundaries (see layout.h)
     uint64_t n_class_segs = 0;
-    for (uint64_t q = L.list_off; q < n_lists; ++q) {
-      const ChunkDesc& d = h.chunks[h.lists[q]];
+    for (uint64_t i = list_off; i < n_lists; ++i) {
+      const ChunkDesc& d = h.chunks[h.lists[i]];
       const uint64_t nb = d.len / kBlockBytes;
       for (uint64_t j = 0; j < nb; j += kSegBlocks) h.seg_start[n_class_segs++] = d.blk_begin + j;
     }
     h.seg_start[n_class_segs] = blk;
     uint64_t k = 0;
-    for (uint64_t w = 0; w < W; ++w) {
-      const uint64_t b0 = h.seg_start[n_class_segs * w / W], b1 = h.seg_start[n_class_segs * (w + 1) / W];
-      WarpDesc& wd = h.warps[n_warps++];
+    for (uint64_t w = 0; w < Wq; ++w) {
+      const uint64_t b0 = h.seg_start[n_class_segs * w / Wq], b1 = h.seg_start[n_class_segs * (w + 1) / Wq];
+      WarpDesc& wd = h.warps[h.slot[q * kMaxWarps + w]];
       std::memset(&wd, 0, sizeof wd);
       wd.blk_begin = b0;
       wd.nblk = b1 - b0;
       wd.rec_base = static_cast<uint32_t>(n_recs);
+      wd.cls = cls;
+      wd.list_off = static_cast<uint32_t>(list_off);
       if (b1 == b0) continue;
       while (b0 >= h.chunks[list[k]].blk_begin + h.chunks[list[k]].len / kBlockBytes) ++k;
       wd.first_chunk = static_cast<uint32_t>(k);
@@ -202,13 +215,13 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
         const uint64_t n = std::min(b1, end) - b;
         if (d.n_recs == 0) d.first_rec = static_cast<uint32_t>(n_recs);
         d.n_recs += 1;
-        h.rec_nblk[n_recs++] = n;  // n_recs <= W per class + chunks <= kMaxRecs
+        h.rec_nblk[n_recs++] = n;  // n_recs <= W + chunks <= kMaxRecs
         b += n;
         if (b == end) ++j;
       }
     }
-    launches[n_launch++] = L;
   }
+  const uint64_t n_warps = n_cls > 0 ? W : 0;
 
   // ---- tables into the scratch, ordered on the caller's stream
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -223,16 +236,16 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
 
   const ChunkDesc* d_chunks = reinterpret_cast<const ChunkDesc*>(scratch + kOffChunks);
   Record* d_recs = reinterpret_cast<Record*>(scratch + kOffRecs);
-  for (int i = 0; i < n_launch; ++i) {
+  if (n_cls > 0) {
     SweepParams sp;
     sp.chunks = d_chunks;
-    sp.warps = reinterpret_cast<const WarpDesc*>(scratch + kOffWarps) + launches[i].warp_off;
-    sp.class_chunks = reinterpret_cast<const uint32_t*>(scratch + kOffLists) + launches[i].list_off;
+    sp.warps = reinterpret_cast<const WarpDesc*>(scratch + kOffWarps);
+    sp.class_chunks = reinterpret_cast<const uint32_t*>(scratch + kOffLists);
     sp.recs = d_recs;
     sp.segs = reinterpret_cast<double*>(scratch + kOffSegs);
     sp.packed = nullptr;
     sp.n_warps = static_cast<uint32_t>(W);
-    e = launch_sweep_fp(launches[i].dtype, launches[i].aligned, sp, n_sm, s);
+    e = launch_sweep_fp_mixed(sp, n_sm, s);
     if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
   }
   FinalizeParams fp;
