@@ -10,7 +10,7 @@ import torch
 import oracle
 from paper_2509_03047_gb300 import synth
 
-from gpu_helpers import expected_mismatch, table_np
+from gpu_helpers import expected_mismatch, odd_tensors, table_np
 
 pytestmark = pytest.mark.gpu
 
@@ -142,6 +142,48 @@ def test_restore_pipelined(where, n_batches):
     ref = src.pack()
     torch.cuda.synchronize()
     assert torch.equal(ref.cpu() if where == "pinned" else ref, staging)
+    assert torch.equal(src.fingerprint(), dst.fingerprint())
+
+
+@pytest.mark.parametrize("offset,chunk,n_batches", [(2, 4096, 5), (4, 12288, 3), (0, 1000, 9)])
+def test_restore_every_class_in_batches(offset, chunk, n_batches):
+    """Batches that hold chunks of every (element type, alignment) class --
+    byte, bf16 and fp32 tensors, some views misaligned -- go through the
+    pipelined restore with its re-sends, both fingerprint tables included."""
+    st = odd_tensors(9, offset)
+    src = fr.Plan(st, chunk, n_batches=n_batches)
+    dst_t = _fresh(st)
+    dst = fr.Plan(dst_t, chunk, n_batches=n_batches)
+    staging = src.new_packed()
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    fa = torch.full((src.n_chunks * 16,), 0xEE, dtype=torch.uint8, device="cuda")
+    fb = torch.full_like(fa, 0xDD)
+    cnt = torch.full((1,), -1, dtype=torch.int64, device="cuda")
+    fr.fr_restore_fp(src.handle, dst.handle, staging, 1, None, cnt, fa, fb, s1, s2)
+    s2.synchronize()
+    assert int(cnt.item()) == 0
+    assert _same(st, dst_t)
+    want = src.fingerprint()
+    torch.cuda.synchronize()
+    assert torch.equal(fa, want) and torch.equal(fb, want)
+
+
+def test_restore_of_tensors_without_a_body():
+    """Every tensor shorter than one 512-byte block: batches with no sweep
+    work at all, only tails."""
+    g = torch.Generator(device="cuda")
+    g.manual_seed(3)
+    st = [torch.randn(int(n), generator=g, device="cuda") for n in (1, 5, 64, 127, 100, 3, 90)]
+    st += [torch.randint(0, 256, (int(n),), generator=g, device="cuda", dtype=torch.uint8) for n in (7, 511, 300)]
+    src = fr.Plan(st, 64, n_batches=4)
+    dst_t = _fresh(st)
+    dst = fr.Plan(dst_t, 64, n_batches=4)
+    staging = src.new_packed()
+    cnt = torch.full((1,), -1, dtype=torch.int64, device="cuda")
+    fr.fr_restore(src.handle, dst.handle, staging, 1, None, cnt)
+    torch.cuda.synchronize()
+    assert int(cnt.item()) == 0
+    assert _same(st, dst_t)
     assert torch.equal(src.fingerprint(), dst.fingerprint())
 
 
