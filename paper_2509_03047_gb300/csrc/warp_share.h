@@ -67,24 +67,15 @@ inline void share_warps(const double* cost, int n, uint64_t W, uint64_t* wc) {
 }
 
 // slot[q * stride + j] = launch-warp index of class q's j-th warp.  Slot i is
-// warp i / n_ctas of CTA i % n_ctas; slots go in order to the class furthest
-// behind its share of the slots so far, which spreads every class evenly over
-// the CTAs.  sum(wc) == W.
+// warp i / n_ctas of CTA i % n_ctas (round robin over the CTAs), and each
+// class takes a run of consecutive slots, so every CTA holds the floor or the
+// ceiling of its share of every class.  sum(wc) == W.
 inline void spread_warps(const uint64_t* wc, int n, uint64_t W, int n_ctas, int warps_per_cta, uint32_t* slot,
                          uint64_t stride) {
-  uint64_t done[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-  for (uint64_t i = 0; i < W; ++i) {
-    int best = -1;
-    double gap = -1e300;
-    for (int q = 0; q < n; ++q) {
-      if (done[q] == wc[q]) continue;
-      const double g = static_cast<double>(wc[q]) * static_cast<double>(i + 1) / static_cast<double>(W) -
-                       static_cast<double>(done[q]);
-      if (g > gap) gap = g, best = q;
-    }
-    slot[best * stride + done[best]] = static_cast<uint32_t>((i % n_ctas) * warps_per_cta + i / n_ctas);
-    ++done[best];
-  }
+  uint64_t i = 0;
+  for (int q = 0; q < n; ++q)
+    for (uint64_t j = 0; j < wc[q] && i < W; ++j, ++i)
+      slot[q * stride + j] = static_cast<uint32_t>((i % n_ctas) * warps_per_cta + i / n_ctas);
 }
 
 }  // namespace frk
