@@ -249,18 +249,18 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
       D.batches.push_back(bi);
       continue;
     }
-    // warps per class, and (mixed) the batch-warp slot of each class's j-th warp
+    // warps per class, and (mixed) slot[q * W + j] = the batch-warp index of
+    // class q's j-th warp
     std::vector<uint64_t> wc(cl.size(), W);
-    std::vector<std::vector<uint64_t>> slot(cl.size());
+    std::vector<uint32_t> slot;
     const uint64_t warp_base = warps.size();
     if (mixed) {
       double cost[6];
       for (size_t q = 0; q < cl.size(); ++q)
         cost[q] = static_cast<double>(class_blocks[cl[q].cls]) * block_weight(cl[q].cls / 2, mix);
       share_warps(cost, static_cast<int>(cl.size()), W, wc.data());
-      std::vector<uint32_t> slots(cl.size() * W);
-      spread_warps(wc.data(), static_cast<int>(cl.size()), W, n_ctas, warps_per_cta, slots.data(), W);
-      for (size_t q = 0; q < cl.size(); ++q) slot[q].assign(slots.begin() + q * W, slots.begin() + q * W + wc[q]);
+      slot.resize(cl.size() * W);
+      spread_warps(wc.data(), static_cast<int>(cl.size()), W, n_ctas, warps_per_cta, slot.data(), W);
       warps.resize(warp_base + W);
       SweepClass sc;
       sc.warp_off = warp_base;
@@ -304,7 +304,7 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
           }
         }
         if (mixed)
-          warps[warp_base + slot[q][w]] = wd;
+          warps[warp_base + slot[q * W + w]] = wd;
         else
           warps.push_back(wd);
       }

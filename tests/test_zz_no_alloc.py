@@ -13,7 +13,7 @@ import torch
 
 from paper_2509_03047_gb300 import synth
 
-from gpu_helpers import assert_tables_match, table_np
+from gpu_helpers import assert_tables_match, odd_tensors, table_np
 
 pytestmark = pytest.mark.gpu
 
@@ -28,7 +28,7 @@ def _static_table(tensors, chunk):
     return out
 
 
-def test_static_entry_point_matches_plan_on_two_calls_in_a_row():
+def test_static_entry_point_matches_plan_on_three_calls_in_a_row():
     # call 1: the tiny workload, with its injected NaNs
     cfg = synth.get_config("tiny")
     a = synth.make_state(cfg, "cuda")
@@ -37,7 +37,9 @@ def test_static_entry_point_matches_plan_on_two_calls_in_a_row():
     base = torch.randn((3 << 20) + 64, device="cuda")
     b = [base[1:1 + 700000], base[800001:800001 + 333333].to(torch.bfloat16).contiguous(),
          base[2000000:2000000 + 1000003], torch.randint(0, 256, (99999,), device="cuda", dtype=torch.uint8)]
-    for tensors, chunk in [(a, cfg.chunk_bytes), (b, 12288)]:
+    # call 3: every (element type, alignment) class, awkward sizes
+    c = odd_tensors(4, 2)
+    for tensors, chunk in [(a, cfg.chunk_bytes), (b, 12288), (c, 4096)]:
         want = fr.Plan(tensors, chunk).fingerprint()
         got = _static_table(tensors, chunk)
         assert got.numel() == want.numel()
