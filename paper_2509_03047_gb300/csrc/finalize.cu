@@ -21,8 +21,11 @@
 //      after the header table; unpack: checks the header against the plan, the
 //      header CRC, the payload CRC and the padding, and writes a verdict.
 //      Pack and unpack-fp also write the table entry when given a table.
-// The verdicts become an ascending id list through a single-CTA ordered
-// compaction, which fr_diff shares with a different predicate.
+// The verdicts become an ascending id list through an ordered compaction --
+// one CTA for up to one tile of ids, a cluster of CTAs sharing their tile
+// counts through distributed shared memory beyond that -- which fr_diff
+// shares with a different predicate.
+#include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
 #include <cstdint>
@@ -528,6 +531,103 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(Pred pred, uin
   }
 }
 
+// The same compaction over a cluster of kCompactCluster CTAs for more than
+// one tile: in round r, CTA k tests tile r * kCompactCluster + k exactly as
+// above, publishes its hit count in its shared memory, and after a cluster
+// barrier reads the other CTAs' counts through distributed shared memory to
+// place its ids after those of the lower tiles.  A second barrier per round
+// keeps a count from being overwritten before every CTA has read it.  Every
+// CTA runs the same number of rounds and reaches every barrier; no global
+// scratch, no atomics deciding positions.
+constexpr int kCompactCluster = 8;
+
+template <class Pred>
+__global__ void __cluster_dims__(kCompactCluster, 1, 1) __launch_bounds__(kCompactThreads)
+    compact_cluster_kernel(Pred pred, uint64_t n, uint32_t* out, uint64_t cap, uint64_t* count, uint32_t* status) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cluster = cg::this_cluster();
+  __shared__ uint32_t warp_tot[kCompactThreads / 32];
+  __shared__ uint32_t tile_tot;     // this CTA's hits this round, read by the whole cluster
+  __shared__ uint64_t round_first;  // this CTA's first output position this round
+  __shared__ uint64_t round_hits;   // the cluster's hits this round
+  const uint32_t rank = cluster.block_rank();
+  const uint32_t tid = threadIdx.x, lane = tid & 31u, warp = tid >> 5;
+  const uint32_t lt = (1u << lane) - 1u;
+  const uint64_t n_tiles = (n + kTile - 1) / kTile;
+  const uint64_t rounds = (n_tiles + kCompactCluster - 1) / kCompactCluster;
+  constexpr uint64_t kStride = static_cast<uint64_t>(kCompactCluster) * kTile;
+  uint64_t base = 0;
+  if (tid == 0 && static_cast<uint64_t>(rank) * kTile < n) {
+    const uint64_t t0 = static_cast<uint64_t>(rank) * kTile;
+    pred.prefetch(t0, n - t0 < kTile ? n - t0 : kTile);
+  }
+  for (uint64_t r = 0; r < rounds; ++r) {
+    const uint64_t t0 = r * kStride + static_cast<uint64_t>(rank) * kTile;  // may lie past n: no hits
+    if (tid == 0 && t0 + kStride < n) pred.prefetch(t0 + kStride, n - (t0 + kStride) < kTile ? n - (t0 + kStride) : kTile);
+    const uint64_t wbase = t0 + static_cast<uint64_t>(warp) * (32 * kPerThread);
+    uint32_t mask[kPerThread];
+    uint32_t total = 0;
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      const uint64_t i = wbase + 32u * j + lane;
+      const bool in = i < n;
+      const bool hit = pred(in ? i : 0);
+      mask[j] = __ballot_sync(kFull, in && hit);
+      total += __popc(mask[j]);
+    }
+    if (lane == 0) warp_tot[warp] = total;
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t w = warp_tot[lane];
+      uint32_t winc = w;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const uint32_t v = __shfl_up_sync(kFull, winc, d);
+        if (lane >= static_cast<uint32_t>(d)) winc += v;
+      }
+      warp_tot[lane] = winc - w;  // exclusive prefix of warp totals
+      if (lane == 31) tile_tot = winc;
+    }
+    cluster.sync();  // every CTA's tile_tot is written and visible
+    if (tid == 0) {
+      uint64_t before = 0, hits = 0;
+      for (uint32_t k = 0; k < static_cast<uint32_t>(kCompactCluster); ++k) {
+        const uint32_t v = *cluster.map_shared_rank(&tile_tot, k);
+        if (k < rank) before += v;
+        hits += v;
+      }
+      round_first = base + before;
+      round_hits = hits;
+    }
+    __syncthreads();
+    uint64_t pos = round_first + warp_tot[warp];
+#pragma unroll
+    for (int j = 0; j < kPerThread; ++j) {
+      if ((mask[j] >> lane) & 1u) {
+        const uint64_t q = pos + __popc(mask[j] & lt);
+        if (q < cap) out[q] = static_cast<uint32_t>(wbase + 32u * j + lane);
+      }
+      pos += __popc(mask[j]);
+    }
+    base += round_hits;
+    cluster.sync();  // every CTA has read the tile counts and round_hits
+  }
+  if (rank == 0 && tid == 0) {
+    *count = base;
+    if (base > cap && status != nullptr) atomicOr(status, kStatusCapacity);
+  }
+}
+
+template <class Pred>
+cudaError_t launch_compact(const Pred& pred, uint64_t n, uint32_t* out, uint64_t cap, uint64_t* count,
+                           uint32_t* status, cudaStream_t s) {
+  if (n > static_cast<uint64_t>(kTile))
+    compact_cluster_kernel<Pred><<<kCompactCluster, kCompactThreads, 0, s>>>(pred, n, out, cap, count, status);
+  else
+    compact_kernel<Pred><<<1, kCompactThreads, 0, s>>>(pred, n, out, cap, count, status);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_finalize(int mode, const FinalizeParams& p, cudaStream_t s) {
@@ -547,15 +647,13 @@ cudaError_t launch_finalize(int mode, const FinalizeParams& p, cudaStream_t s) {
 
 cudaError_t launch_compact_flags(const uint8_t* flags, uint64_t n, uint32_t* out, uint64_t cap,
                                  uint64_t* count, uint32_t* status, cudaStream_t s) {
-  compact_kernel<FlagPred><<<1, kCompactThreads, 0, s>>>(FlagPred{flags}, n, out, cap, count, status);
-  return cudaGetLastError();
+  return launch_compact(FlagPred{flags}, n, out, cap, count, status, s);
 }
 
 cudaError_t launch_diff(const FpEntry* a, const FpEntry* b, uint64_t n, uint32_t* out, uint64_t cap,
                         uint64_t* count, cudaStream_t s) {
   DiffPred pred{reinterpret_cast<const uint4*>(a), reinterpret_cast<const uint4*>(b)};
-  compact_kernel<DiffPred><<<1, kCompactThreads, 0, s>>>(pred, n, out, cap, count, nullptr);
-  return cudaGetLastError();
+  return launch_compact(pred, n, out, cap, count, nullptr, s);
 }
 
 }  // namespace frk
