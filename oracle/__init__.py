@@ -117,6 +117,9 @@ def _bind(L: ctypes.CDLL) -> ctypes.CDLL:
     L.or_unpack_verify.argtypes = [ctypes.POINTER(ctypes.c_void_p), u64p, u32p, c_u64, c_u64,
                                    ctypes.c_void_p, c_u64, u32p, c_u64, u64p]
     L.or_unpack_verify.restype = ctypes.c_int
+    L.or_verify_chunk.argtypes = [ctypes.POINTER(_OrChunk), c_u64, ctypes.c_void_p, ctypes.c_void_p,
+                                  ctypes.c_void_p, c_u64]
+    L.or_verify_chunk.restype = ctypes.c_int
     L.or_diff.argtypes = [ctypes.c_void_p, ctypes.c_void_p, c_u64, u32p, c_u64]
     L.or_diff.restype = c_u64
     return L
@@ -211,6 +214,22 @@ def header(chunk, chunk_id: int, fp) -> bytes:
     h = np.zeros(64, dtype=np.uint8)
     lib().or_header(ctypes.byref(ch), chunk_id, ctypes.byref(f), _ptr(h))
     return h.tobytes()
+
+
+def verify_chunk(chunk, chunk_id: int, header_bytes, payload_and_padding, gap=None) -> bool:
+    """The oracle's unpack verdict for one chunk (True: it fails a check).
+    `payload_and_padding` holds the chunk's payload and its zero padding
+    (len rounded up to 256 bytes); `gap` the zero gap after the header table,
+    passed for the last chunk only."""
+    ch = _OrChunk(int(chunk["tensor_idx"]), int(chunk["dtype"]), int(chunk["tensor_off"]),
+                  int(chunk["len"]), int(chunk["payload_off"]))
+    h = _as_u8(header_bytes)
+    p = _as_u8(payload_and_padding)
+    assert h.size == HEADER_BYTES
+    assert p.size == (int(chunk["len"]) + PAYLOAD_ALIGN - 1) // PAYLOAD_ALIGN * PAYLOAD_ALIGN
+    g = _as_u8(gap) if gap is not None else np.zeros(0, dtype=np.uint8)
+    return bool(lib().or_verify_chunk(ctypes.byref(ch), chunk_id, _ptr(h), _ptr(p) or None,
+                                      _ptr(g) or None, g.size))
 
 
 # ---------------------------------------------------------------- whole state

@@ -284,6 +284,36 @@ int or_pack(const uint8_t* const* tensors, const uint64_t* nbytes,
   return OR_OK;
 }
 
+/* The checks of unpack_verify on one chunk: the header CRC, every addressing
+ * field against the receiver's own plan, the payload CRC, the zero padding,
+ * and (last chunk only) the zero gap after the header table.  Returns 1 if
+ * any check fails. */
+int or_verify_chunk(const or_chunk* ch, uint64_t chunk_id, const uint8_t* h,
+                    const uint8_t* payload, const uint8_t* gap, uint64_t gap_len) {
+  int bad = 0;
+  /* 1. the header protects itself */
+  if (load_le32(h + 60) != or_crc32c(h, 60)) bad = 1;
+  /* 2. every addressing field must equal the receiver's own plan */
+  if (load_le32(h + 0) != OR_MAGIC) bad = 1;
+  if (load_le16(h + 4) != OR_VERSION) bad = 1;
+  if (load_le16(h + 6) != ch->dtype) bad = 1;
+  if (load_le64(h + 8) != chunk_id) bad = 1;
+  if (load_le32(h + 16) != ch->tensor_idx) bad = 1;
+  if (load_le64(h + 24) != ch->tensor_off) bad = 1;
+  if (load_le64(h + 32) != ch->len) bad = 1;
+  if (load_le64(h + 40) != ch->payload_off) bad = 1;
+  /* 3. the payload must match the CRC the header carries */
+  if (or_crc32c(payload, ch->len) != load_le32(h + 20)) bad = 1;
+  /* 4. the padding after the payload must be zero */
+  uint64_t pad_end = align_up(ch->len, OR_PAYLOAD_ALIGN);
+  for (uint64_t i = ch->len; i < pad_end; ++i)
+    if (payload[i] != 0) bad = 1;
+  /* the gap after the header table (passed for the last chunk only) */
+  for (uint64_t i = 0; i < gap_len; ++i)
+    if (gap[i] != 0) bad = 1;
+  return bad;
+}
+
 int or_unpack_verify(uint8_t* const* tensors, const uint64_t* nbytes,
                      const uint32_t* dtypes, uint64_t n_tensors, uint64_t chunk_bytes,
                      const uint8_t* src, uint64_t src_bytes,
@@ -295,36 +325,16 @@ int or_unpack_verify(uint8_t* const* tensors, const uint64_t* nbytes,
     free(chunks);
     return OR_ERR_BUFFER_TOO_SMALL;
   }
+  uint64_t gap_begin = count * OR_HEADER_BYTES;
+  uint64_t gap_end = align_up(count * OR_HEADER_BYTES, OR_PAYLOAD_ALIGN);
   uint64_t found = 0;
   for (uint64_t c = 0; c < count; ++c) {
     const or_chunk* ch = &chunks[c];
-    const uint8_t* h = src + c * OR_HEADER_BYTES;
     const uint8_t* payload = src + ch->payload_off;
-    int bad = 0;
-
-    /* 1. the header protects itself */
-    if (load_le32(h + 60) != or_crc32c(h, 60)) bad = 1;
-    /* 2. every addressing field must equal the receiver's own plan */
-    if (load_le32(h + 0) != OR_MAGIC) bad = 1;
-    if (load_le16(h + 4) != OR_VERSION) bad = 1;
-    if (load_le16(h + 6) != ch->dtype) bad = 1;
-    if (load_le64(h + 8) != c) bad = 1;
-    if (load_le32(h + 16) != ch->tensor_idx) bad = 1;
-    if (load_le64(h + 24) != ch->tensor_off) bad = 1;
-    if (load_le64(h + 32) != ch->len) bad = 1;
-    if (load_le64(h + 40) != ch->payload_off) bad = 1;
-    /* 3. the payload must match the CRC the header carries */
-    if (or_crc32c(payload, ch->len) != load_le32(h + 20)) bad = 1;
-    /* 4. the padding after the payload must be zero */
-    uint64_t pad_end = ch->payload_off + align_up(ch->len, OR_PAYLOAD_ALIGN);
-    for (uint64_t i = ch->payload_off + ch->len; i < pad_end; ++i)
-      if (src[i] != 0) bad = 1;
     /* the gap after the header table belongs to the last chunk */
-    if (c + 1 == count) {
-      uint64_t gap_end = align_up(count * OR_HEADER_BYTES, OR_PAYLOAD_ALIGN);
-      for (uint64_t i = count * OR_HEADER_BYTES; i < gap_end; ++i)
-        if (src[i] != 0) bad = 1;
-    }
+    int last = (c + 1 == count);
+    int bad = or_verify_chunk(ch, c, src + c * OR_HEADER_BYTES, payload,
+                              last ? src + gap_begin : 0, last ? gap_end - gap_begin : 0);
 
     /* the payload is copied to the plan's destination whatever the verdict */
     memcpy(tensors[ch->tensor_idx] + ch->tensor_off, payload, (size_t)ch->len);

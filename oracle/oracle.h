@@ -118,6 +118,17 @@ int or_pack(const uint8_t* const* tensors, const uint64_t* nbytes,
             const uint32_t* dtypes, uint64_t n_tensors, uint64_t chunk_bytes,
             uint8_t* dst, uint64_t dst_bytes);
 
+/* The verdict of unpack_verify for one chunk: 1 if it fails any check.
+ *   ch, chunk_id  the receiver's own plan entry for the chunk;
+ *   h             the chunk's 64-byte header in the packed buffer;
+ *   payload       its payload followed by its zero padding
+ *                 (ch->len rounded up to OR_PAYLOAD_ALIGN bytes);
+ *   gap, gap_len  the zero gap between the header table and the first
+ *                 payload, which belongs to the last chunk: pass it for the
+ *                 last chunk only (else NULL, 0). */
+int or_verify_chunk(const or_chunk* ch, uint64_t chunk_id, const uint8_t* h,
+                    const uint8_t* payload, const uint8_t* gap, uint64_t gap_len);
+
 /* Always copies every payload to its plan destination; lists, ascending,
  * the chunks that fail any check.  *n_mismatch gets the true count; at most
  * `cap` ids are written. */

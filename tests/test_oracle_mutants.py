@@ -30,12 +30,12 @@ MUTANTS = {
     "header_crc_span": ("store_le32(h + 60, or_crc32c(h, 60));", "store_le32(h + 60, or_crc32c(h, 56));"),
     "payload_align": ("off += align_up(len, OR_PAYLOAD_ALIGN);", "off += align_up(len, 128);"),
     "tail_length": ("if (len > chunk_bytes) len = chunk_bytes;", "if (len >= chunk_bytes) len = chunk_bytes - 4;"),
-    "no_padding_check": ("for (uint64_t i = ch->payload_off + ch->len; i < pad_end; ++i)\n      if (src[i] != 0) bad = 1;",
-                         "for (uint64_t i = ch->payload_off + ch->len; i < pad_end; ++i)\n      if (0) bad = 1;"),
-    "no_gap_check": ("for (uint64_t i = count * OR_HEADER_BYTES; i < gap_end; ++i)\n        if (src[i] != 0) bad = 1;",
-                     "for (uint64_t i = count * OR_HEADER_BYTES; i < gap_end; ++i)\n        if (0) bad = 1;"),
+    "no_padding_check": ("for (uint64_t i = ch->len; i < pad_end; ++i)\n    if (payload[i] != 0) bad = 1;",
+                         "for (uint64_t i = ch->len; i < pad_end; ++i)\n    if (0) bad = 1;"),
+    "no_gap_check": ("for (uint64_t i = 0; i < gap_len; ++i)\n    if (gap[i] != 0) bad = 1;",
+                     "for (uint64_t i = 0; i < gap_len; ++i)\n    if (0) bad = 1;"),
     "no_offset_check": ("if (load_le64(h + 24) != ch->tensor_off) bad = 1;", ""),
-    "no_chunk_id_check": ("if (load_le64(h + 8) != c) bad = 1;", ""),
+    "no_chunk_id_check": ("if (load_le64(h + 8) != chunk_id) bad = 1;", ""),
     "copy_only_good": ("memcpy(tensors[ch->tensor_idx] + ch->tensor_off, payload, (size_t)ch->len);",
                        "if (!bad) memcpy(tensors[ch->tensor_idx] + ch->tensor_off, payload, (size_t)ch->len);"),
     "diff_crc_only": ("if (memcmp(&a[c], &b[c], sizeof(or_fp)) != 0) {", "if (memcmp(&a[c], &b[c], 4) != 0) {"),

@@ -276,3 +276,31 @@ def test_swapped_headers_are_flagged(orc):
     bad[64 * 2: 64 * 3], bad[64 * 5: 64 * 6] = buf[64 * 5: 64 * 6], buf[64 * 2: 64 * 3]
     rc, ids, n = orc.unpack_verify(_fresh_dst(arrs), dts, CHUNK, bad)
     assert list(ids) == [2, 5]
+
+
+def test_per_chunk_verdicts_match_where_the_flips_landed(orc):
+    """verify_chunk, given each chunk's header, payload + padding and (last
+    chunk) the table gap, sliced by the independent layout restatement, flags
+    exactly the owners of the flipped bytes -- the whole-buffer call's result
+    chunk by chunk, so tests can spread the chunks over host threads."""
+    arrs, dts = adversarial_state(7)
+    buf = orc.pack(arrs, dts, CHUNK)
+    chunks, offs, size = py_plan([a.size for a in arrs], CHUNK)
+    ochunks, _ = orc.plan([a.size for a in arrs], dts, CHUNK)
+    C = len(chunks)
+    gap = (64 * C, a256(64 * C))
+    assert gap[1] > gap[0]  # this layout has a gap for the probe below
+    cases = [np.zeros(0, dtype=np.int64), np.array([gap[0] * 8 + 2])]
+    cases += [synth.flip_positions(size, k, seed=100 + k) for k in (1, 3, 17, 60)]
+    for pos in cases:
+        bad = buf.copy()
+        for p in pos:
+            bad[p // 8] ^= np.uint8(1 << (p % 8))
+        want = sorted({owner_of_byte(int(p) // 8, chunks, offs) for p in pos})
+        got = [c for c in range(C)
+               if orc.verify_chunk(ochunks[c], c, bad[64 * c: 64 * c + 64],
+                                   bad[offs[c]: offs[c] + a256(chunks[c][2])],
+                                   bad[gap[0]: gap[1]] if c == C - 1 else None)]
+        assert got == want
+        rc, ids, n = orc.unpack_verify(_fresh_dst(arrs), dts, CHUNK, bad)
+        assert list(ids) == got
