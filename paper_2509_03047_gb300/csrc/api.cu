@@ -119,6 +119,22 @@ fr_status cuda_fail(cudaError_t e, const char* where) {
   return FR_ERR_CUDA;
 }
 
+}  // namespace
+
+// The other translation units' entry points report through the same
+// thread-local message.
+fr_status frk::report_invalid(const char* where, const char* what) {
+  set_err("%s: invalid argument: %s", where, what);
+  return FR_ERR_INVALID_ARG;
+}
+
+fr_status frk::report_cuda(const char* where, cudaError_t e) {
+  set_err("%s: %s", where, cudaGetErrorString(e));
+  return FR_ERR_CUDA;
+}
+
+namespace {
+
 uint64_t elem_bytes(uint32_t dt) { return dt == kDtF32 ? 4 : (dt == kDtBf16 ? 2 : 1); }
 
 // Kernels are configured once per device.

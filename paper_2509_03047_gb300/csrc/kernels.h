@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include "layout.h"
+#include "../../include/flashrec.h"
 
 namespace frk {
 
@@ -109,5 +110,10 @@ cudaError_t launch_compact_flags(const uint8_t* flags, uint64_t n, uint32_t* out
 // Ascending ids of the differing 16-byte entries, first `cap`, true count.
 cudaError_t launch_diff(const FpEntry* a, const FpEntry* b, uint64_t n, uint32_t* out, uint64_t cap,
                         uint64_t* count, cudaStream_t s);
+
+// Set the calling thread's fr_last_error message and return the status
+// (FR_ERR_INVALID_ARG with `what`, FR_ERR_CUDA with the CUDA error's text).
+fr_status report_invalid(const char* where, const char* what);
+fr_status report_cuda(const char* where, cudaError_t e);
 
 }  // namespace frk

@@ -77,20 +77,20 @@ uint8_t* g_dev_ptr[kMaxDevices] = {};
 
 uint64_t elem_bytes(uint32_t dt) { return dt == kDtF32 ? 4 : (dt == kDtBf16 ? 2 : 1); }
 
-// `what` documents the reason at the call site; the status is what returns.
-fr_status fail(fr_status s, const char* what) {
-  (void)what;
-  return s;
-}
+// Records the reason for fr_last_error and returns the status.
+constexpr const char* kWhere = "fr_fingerprint_static";
+fr_status fail(const char* what) { return report_invalid(kWhere, what); }
+fr_status fail(cudaError_t e) { return report_cuda(kWhere, e); }
 
 fr_status setup_device(int dev, uint8_t** out) {
-  if (dev < 0 || dev >= kMaxDevices) return fail(FR_ERR_INVALID_ARG, "device index out of range");
+  if (dev < 0 || dev >= kMaxDevices) return fail("device index out of range");
   if (g_dev_ptr[dev] == nullptr) {
     void* ptr = nullptr;
     cudaError_t e = cudaGetSymbolAddress(&ptr, g_static_scratch);
-    if (e != cudaSuccess || ptr == nullptr) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+    if (e != cudaSuccess) return fail(e);
+    if (ptr == nullptr) return fail("the scratch array has no device address");
     e = configure_sweep_fp();
-    if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+    if (e != cudaSuccess) return fail(e);
     g_dev_ptr[dev] = static_cast<uint8_t*>(ptr);
   }
   *out = g_dev_ptr[dev];
@@ -101,17 +101,18 @@ fr_status setup_device(int dev, uint8_t** out) {
 
 extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes,
                                            fr_fp* out_dev, void* stream) {
-  if (n_tensors > 0 && tensors == nullptr) return fail(FR_ERR_INVALID_ARG, "tensors is null");
-  if (chunk_bytes == 0 || chunk_bytes % 4 != 0) return fail(FR_ERR_INVALID_ARG, "chunk_bytes must be a positive multiple of 4");
+  if (n_tensors > 0 && tensors == nullptr) return fail("tensors is null");
+  if (n_tensors >= (1ull << 32)) return fail("more than 2^32 - 1 tensors");
+  if (chunk_bytes == 0 || chunk_bytes % 4 != 0) return fail("chunk_bytes must be a positive multiple of 4");
   uint64_t n_chunks = 0;
   for (uint64_t t = 0; t < n_tensors; ++t) {
     const fr_tensor& x = tensors[t];
-    if (x.dtype > FR_DT_F32 || x.flags != 0) return fail(FR_ERR_INVALID_ARG, "bad dtype or flags");
-    if (x.nbytes % elem_bytes(x.dtype) != 0) return fail(FR_ERR_INVALID_ARG, "nbytes is not a multiple of the element size");
-    if (x.nbytes > 0 && x.ptr == nullptr) return fail(FR_ERR_INVALID_ARG, "tensor pointer is null");
-    if (x.nbytes >= (1ull << 47)) return fail(FR_ERR_INVALID_ARG, "tensor too large");
+    if (x.dtype > FR_DT_F32 || x.flags != 0) return fail("bad dtype or flags");
+    if (x.nbytes % elem_bytes(x.dtype) != 0) return fail("nbytes is not a multiple of the element size");
+    if (x.nbytes > 0 && x.ptr == nullptr) return fail("tensor pointer is null");
+    if (x.nbytes >= (1ull << 47)) return fail("tensor too large");
     n_chunks += (x.nbytes + chunk_bytes - 1) / chunk_bytes;
-    if (n_chunks > kMaxChunks) return fail(FR_ERR_INVALID_ARG, "more chunks than FR_STATIC_MAX_CHUNKS");
+    if (n_chunks > kMaxChunks) return fail("more chunks than FR_STATIC_MAX_CHUNKS");
   }
   uint64_t n_segs = 0;
   for (uint64_t t = 0; t < n_tensors; ++t)
@@ -119,18 +120,18 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
       const uint64_t len = std::min<uint64_t>(chunk_bytes, tensors[t].nbytes - off);
       n_segs += (len / kBlockBytes + kSegBlocks - 1) / kSegBlocks;
     }
-  if (n_segs > kMaxSegs) return fail(FR_ERR_INVALID_ARG, "more sum segments than FR_STATIC_MAX_SEGMENTS");
+  if (n_segs > kMaxSegs) return fail("more sum segments than FR_STATIC_MAX_SEGMENTS");
   if (n_chunks == 0) return FR_OK;
-  if (out_dev == nullptr) return fail(FR_ERR_INVALID_ARG, "out_dev is null");
+  if (out_dev == nullptr) return fail("out_dev is null");
 
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+  if (e != cudaSuccess) return fail(e);
   int n_sm = 0;
   e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
-  if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+  if (e != cudaSuccess) return fail(e);
   const uint64_t W = static_cast<uint64_t>(n_sm) * sweep_warps(kModeFingerprint);
-  if (W > kMaxWarps) return fail(FR_ERR_INVALID_ARG, "GPU has more SMs than the static tables hold");
+  if (W > kMaxWarps) return fail("GPU has more SMs than the static tables hold");
 
   std::lock_guard<std::mutex> lk(g_mu);
   uint8_t* scratch = nullptr;
@@ -232,7 +233,7 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
     e = cudaMemcpyAsync(scratch + kOffWarps, h.warps, n_warps * sizeof(WarpDesc), cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess && n_recs)
     e = cudaMemcpyAsync(scratch + kOffRecNblk, h.rec_nblk, n_recs * sizeof(uint64_t), cudaMemcpyHostToDevice, s);
-  if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+  if (e != cudaSuccess) return fail(e);
 
   const ChunkDesc* d_chunks = reinterpret_cast<const ChunkDesc*>(scratch + kOffChunks);
   Record* d_recs = reinterpret_cast<Record*>(scratch + kOffRecs);
@@ -246,7 +247,7 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
     sp.packed = nullptr;
     sp.n_warps = static_cast<uint32_t>(W);
     e = launch_sweep_fp_mixed(sp, n_sm, s);
-    if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+    if (e != cudaSuccess) return fail(e);
   }
   FinalizeParams fp;
   fp.chunks = d_chunks;
@@ -263,6 +264,6 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
   fp.out_fp = reinterpret_cast<FpEntry*>(out_dev);
   fp.flags = nullptr;
   e = launch_finalize(kModeFingerprint, fp, s);
-  if (e != cudaSuccess) return fail(FR_ERR_CUDA, cudaGetErrorString(e));
+  if (e != cudaSuccess) return fail(e);
   return FR_OK;
 }
