@@ -150,6 +150,20 @@ class ClockSampler:
 
 # ---------------------------------------------------------------- helpers
 
+def repo_libraries_loaded():
+    """Shared objects of this repository mapped into the process."""
+    found = set()
+    try:
+        with open("/proc/self/maps") as f:
+            for line in f:
+                path = line.split()[-1] if line.strip() else ""
+                if path.startswith(ROOT) and ".so" in path:
+                    found.add(os.path.relpath(path, ROOT))
+    except OSError:
+        pass
+    return sorted(found)
+
+
 def measured_peak():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -433,30 +447,26 @@ def run_flashrec(args):
             s_dst.synchronize()
             return int(nmis.item()), int(ndiv.item())
 
-        restore_step()
-        barrier()
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        for _ in range(args.e2e_steps):
-            e2e_found = restore_step()
-        torch.cuda.synchronize()
-        t_e2e = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
+        def sample(fn):
+            """Per-step wall times of `fn` (each step ends by reading its result on
+            the host): (mean, median, best, the last step's result)."""
+            fn()
+            barrier()
+            torch.cuda.synchronize()
+            ts, res = [], None
+            for _ in range(args.e2e_steps):
+                t0 = time.perf_counter()
+                res = fn()
+                ts.append(time.perf_counter() - t0)
+            torch.cuda.synchronize()
+            return (max_over_ranks(sum(ts) / len(ts), dev), max_over_ranks(statistics.median(ts), dev),
+                    max_over_ranks(min(ts), dev), res)
+
+        t_e2e, med_e2e, best_e2e, e2e_found = sample(restore_step)
         # (b) for comparison: the same restore with separate fingerprint sweeps
-        restore_step_unfused()
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        for _ in range(args.e2e_steps):
-            restore_step_unfused()
-        torch.cuda.synchronize()
-        t_unfused = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
+        t_unfused, med_unfused, best_unfused, _ = sample(restore_step_unfused)
         # (c) for comparison: whole-buffer pack, then whole-buffer unpack
-        step(buf=host_buf, sync_counts=True)
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        for _ in range(args.e2e_steps):
-            step(buf=host_buf, sync_counts=True)
-        torch.cuda.synchronize()
-        t_serial = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, dev)
+        t_serial, med_serial, best_serial, _ = sample(lambda: step(buf=host_buf, sync_counts=True))
         # (d) the bound: the host link's copy engines moving P/2 bytes each way
         # at once (64 MiB pieces, two streams, disjoint halves of the buffers)
         half, piece = P // 2, 64 << 20
@@ -471,36 +481,58 @@ def run_flashrec(args):
             torch.cuda.synchronize()
 
         link_step()
-        t_link = float("inf")
-        for _ in range(5):  # the host link's rate varies from call to call: best of 5
+        t_links = []
+        for _ in range(5):  # the host link's rate varies from call to call
             t0 = time.perf_counter()
             link_step()
-            t_link = min(t_link, time.perf_counter() - t0)
+            t_links.append(time.perf_counter() - t0)
+        t_link = min(t_links)
         link_gbs = half / t_link / 1e9
         restore_gbs = P / t_e2e / 1e9
+
+        def ms(x):
+            return round(x * 1e3, 2)
         e2e = {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_e2e / 1e9, dev), 2), "unit": "GB/s",
-               "h2d_bytes_per_step": P, "d2h_bytes_per_step": P + 16, "ms_per_step": round(t_e2e * 1e3, 2),
+               "h2d_bytes_per_step": P, "d2h_bytes_per_step": P + 16, "ms_per_step": ms(t_e2e),
+               "ms_median": ms(med_e2e), "ms_best": ms(best_e2e), "steps": args.e2e_steps,
+               "value_median": round(sum_over_ranks(SWEEPS_PER_STEP * S / med_e2e / 1e9, dev), 2),
                "transfer": "pinned host buffer over NVLink-C2C; fr_restore_fp with %d batches, pack and unpack "
                            "on two streams, both fingerprint tables from the same sweeps, 1 re-send round, then "
                            "fr_diff; no injected flips" % bs.n_batches,
                "unfused": {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_unfused / 1e9, dev), 2),
-                           "ms_per_step": round(t_unfused * 1e3, 2),
+                           "ms_per_step": ms(t_unfused), "ms_median": ms(med_unfused), "ms_best": ms(best_unfused),
                            "how": "fr_fingerprint, fr_restore, fr_fingerprint, fr_diff"},
                "found": {"mismatching_chunks": e2e_found[0], "diverged_chunks": e2e_found[1]},
                "link": {"copy_engines_each_way_gbs": round(link_gbs, 1),
+                        "copy_engines_median_gbs": round(half / statistics.median(t_links) / 1e9, 1),
                         "restore_each_way_gbs": round(restore_gbs, 1), "frac": round(restore_gbs / link_gbs, 4),
+                        "frac_median": round((P / med_e2e) / (half / statistics.median(t_links)), 4),
                         "how": "cudaMemcpyAsync of P/2 bytes device->host and P/2 host->device at once, 64 MiB "
-                               "pieces on two streams, pinned host memory, best of 5; the restore moves P each way"},
+                               "pieces on two streams, pinned host memory, best and median of 5; the restore "
+                               "moves P each way"},
                "serial": {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_serial / 1e9, dev), 2),
-                          "ms_per_step": round(t_serial * 1e3, 2),
+                          "ms_per_step": ms(t_serial), "ms_median": ms(med_serial), "ms_best": ms(best_serial),
                           "how": "fr_pack to the host buffer, then fr_unpack_verify from it, with the flips"}}
         bs.close()
         bd.close()
-        del host_buf
+        del host_buf, bs, bd
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(cfg, src, args.cpu_sample_gb)
+
+    # the other workloads, one at a time, with this state's buffers freed first
+    workloads = None
+    if ws == 1 and args.workloads:
+        plan_s.close()
+        plan_d.close()
+        del src, dst, packed, tab_s, tab_d, plan_s, plan_d
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        held = torch.cuda.memory_allocated(dev)
+        if held > (1 << 30):
+            raise RuntimeError("%d bytes of the headline workload are still held" % held)
+        workloads = time_workloads([w for w in args.workloads.split(",") if w], dev, args.workload_reps, local)
 
     if rank == 0:
         out = {"metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
@@ -515,11 +547,94 @@ def run_flashrec(args):
                           "parallelism": "replicas only (%d independent rank%s)" % (ws, "s" if ws > 1 else ""),
                           "value_def": "4 sweeps x state bytes / step time"},
                "calls": calls, "roofline": roofline, "fused_step": fused, "graph_step": graph, "e2e": e2e,
-               "cpu_baseline": cpu,
+               "cpu_baseline": cpu, "workloads": workloads,
                "gpu_launches": launches_per_step * args.steps, "clocks": clk}
         print(json.dumps(out))
-    plan_s.close()
-    plan_d.close()
+    if workloads is None:
+        plan_s.close()
+        plan_d.close()
+
+
+def time_workloads(names, dev, reps, gpu_index, warmup=3):
+    """Per-call times of fingerprint, pack, unpack_verify and diff on each named
+    workload: the state is generated, its faults injected, every call timed
+    `reps` times with CUDA events on the launching stream after `warmup`
+    untimed calls, and everything freed before the next workload.  States
+    smaller than 1 GiB have L2 (129 MB) flushed by a 256 MiB write before every
+    timed call; larger ones stream far more than L2 holds."""
+    import torch
+
+    from paper_2509_03047_gb300 import flashrec as fr
+    from paper_2509_03047_gb300 import synth
+
+    peak, peak_kind = measured_peak()
+    stream = torch.cuda.current_stream()
+    flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    clocks = ClockSampler(gpu_index)
+    clocks.start()
+    out = {"peak_gbs": peak, "peak_source": peak_kind, "reps": reps, "warmup": warmup}
+    for name in names:
+        t_setup = time.perf_counter()
+        cfg = synth.get_config(name)
+        src = synth.make_state(cfg, dev)
+        nan_pos = synth.inject_nonfinite(cfg, src)
+        dst = [torch.empty_like(t) for t in src]
+        ps, pd = fr.Plan(src, cfg.chunk_bytes), fr.Plan(dst, cfg.chunk_bytes)
+        S, C, P = ps.state_bytes, ps.n_chunks, ps.packed_bytes
+        packed, tab_s, tab_d = ps.new_packed(), ps.new_table(), pd.new_table()
+        mism = torch.empty(max(C, 1), dtype=torch.int32, device=dev)
+        nmis = torch.empty(1, dtype=torch.int64, device=dev)
+        div = torch.empty(max(C, 1), dtype=torch.int32, device=dev)
+        ndiv = torch.empty(1, dtype=torch.int64, device=dev)
+        flush = S < (1 << 30)
+        torch.cuda.synchronize()
+        t_setup = time.perf_counter() - t_setup
+
+        def timed(fn):
+            for _ in range(warmup):
+                fn()
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(reps)]
+            for i, (a, b) in enumerate(evs):
+                if flush:
+                    flush_buf.fill_(i & 0xFF)
+                a.record(stream)
+                fn()
+                b.record(stream)
+            torch.cuda.synchronize()
+            return sorted(a.elapsed_time(b) for a, b in evs)
+
+        t_fp = timed(lambda: fr.fr_fingerprint(ps.handle, tab_s, stream))
+        t_pack = timed(lambda: fr.fr_pack(ps.handle, packed, stream))
+        flips = synth.flip_positions(P, cfg.flips, cfg.seed)
+        synth.apply_flips(packed, flips)
+        t_unpack = timed(lambda: fr.fr_unpack_verify(pd.handle, packed, mism, nmis, stream))
+        fr.fr_fingerprint(pd.handle, tab_d, stream)
+        t_diff = timed(lambda: fr.fr_diff(tab_s, tab_d, C, div, ndiv, stream))
+        found = {"mismatching_chunks": int(nmis.item()), "diverged_chunks": int(ndiv.item())}
+        alg = {"fingerprint": S + 16 * C, "pack": S + P, "unpack_verify": P + S + 4 * C}
+        calls = {}
+        for k, ts in (("fingerprint", t_fp), ("pack", t_pack), ("unpack_verify", t_unpack)):
+            med, best = statistics.median(ts), ts[0]
+            calls[k] = {"ms_median": round(med, 4), "ms_best": round(best, 4),
+                        "ms_mean": round(sum(ts) / len(ts), 4),
+                        "state_gbs": round(S / (med * 1e-3) / 1e9, 1), "alg_bytes": alg[k],
+                        "achieved_gbs": round(alg[k] / (med * 1e-3) / 1e9, 1),
+                        "frac": round(alg[k] / (med * 1e-3) / 1e9 / peak, 4),
+                        "frac_best": round(alg[k] / (best * 1e-3) / 1e9 / peak, 4)}
+        calls["diff"] = {"us_median": round(statistics.median(t_diff) * 1e3, 2), "alg_bytes": 32 * C}
+        out[name] = {"state_bytes": S, "chunk_bytes": cfg.chunk_bytes, "n_chunks": C, "packed_bytes": P,
+                     "tensors": len(src), "faults": {"nonfinite": int(nan_pos.size), "bit_flips": int(flips.size)},
+                     "found": found, "calls": calls, "setup_s": round(t_setup, 1),
+                     "l2": ("L2 flushed (256 MiB write) before every timed call" if flush else
+                            "state %.1f GB streams far more than the 129 MB L2; no flush" % (S / 1e9))}
+        ps.close()
+        pd.close()
+        del src, dst, packed, tab_s, tab_d, mism, div, ps, pd
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+    out["clocks"] = clocks.stop()
+    return out
 
 
 # ---------------------------------------------------------------- the oracle
@@ -581,8 +696,8 @@ def run_reference(args):
     bounded slice of the same workload generated on the host."""
     import torch
 
+    import oracle
     from paper_2509_03047_gb300 import synth
-    from paper_2509_03047_gb300.flashrec import FR_DT_BF16, FR_DT_F32
 
     ws, rank, _ = dist_env()
     if rank != 0:
@@ -600,7 +715,7 @@ def run_reference(args):
         specs = cfg.buffer_specs()
         state = [torch.randn(specs[i][2] // 4, generator=synth._gen("cpu", cfg.seed, i, 9)) for i in idx]
     host = [t.view(torch.uint8).reshape(-1).numpy() for t in state]
-    dts = [FR_DT_BF16 if t.dtype == torch.bfloat16 else FR_DT_F32 for t in state]
+    dts = [oracle.DT_BF16 if t.dtype == torch.bfloat16 else oracle.DT_F32 for t in state]
     for _ in range(args.warmup):
         oracle_sample(cfg, host, dts)
     times = [oracle_sample(cfg, host, dts) for _ in range(args.steps)]
@@ -616,7 +731,10 @@ def run_reference(args):
            "config": {"workload": args.config, "sample_bytes": tot, "chunk_bytes": cfg.chunk_bytes,
                       "value_def": "4 sweeps x state bytes / step time"},
            "cpu_baseline": cpu,
-           "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+           "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+           "native_libraries": repo_libraries_loaded()}
+    if any("libflashrec" in x for x in out["native_libraries"]):
+        raise RuntimeError("the reference arm must not load the product library")
     print(json.dumps(out))
 
 
@@ -627,12 +745,15 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["flashrec", "reference"], default="flashrec")
     ap.add_argument("--config", default=DEFAULT_CONFIG)
-    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--batches", type=int, default=16)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-gb", type=float, default=1.0)
     ap.add_argument("--graph", action="store_true", help="also time the fused step replayed from a CUDA graph")
+    ap.add_argument("--workloads", default="tiny,gpt2s,l8b_tp8,zero_frag,zero_frag4g",
+                    help="comma-separated workloads timed per call after the headline step ('' for none)")
+    ap.add_argument("--workload-reps", type=int, default=10)
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "flashrec":
         ap.error("at least 3 warm-up steps")
