@@ -9,6 +9,53 @@ from paper_2509_03047_gb300 import synth
 
 SUMSQ_RTOL = 1e-9  # the fp64 sums of squares agree within 1e-9 relative
 
+# Every output buffer a test hands the library is followed by GUARD_BYTES of
+# GUARD_FILL; after the call the guard must be intact, so a kernel writing
+# past the end of an output is caught (compute-sanitizer is not available).
+GUARD_BYTES = 4096
+GUARD_FILL = 0x5A
+
+
+class Guarded:
+    """A uint8 output buffer of `nbytes` followed by a guard region."""
+
+    def __init__(self, nbytes, device="cuda", pinned=False, fill=GUARD_FILL):
+        self.nbytes = int(nbytes)
+        self.fill = fill
+        if pinned:
+            self.whole = torch.empty(self.nbytes + GUARD_BYTES, dtype=torch.uint8, pin_memory=True)
+            self.whole.fill_(fill)
+        else:
+            self.whole = torch.full((self.nbytes + GUARD_BYTES,), fill, dtype=torch.uint8, device=device)
+        self.buf = self.whole[: self.nbytes]
+
+    def view(self, dtype):
+        return self.buf.view(dtype) if self.nbytes else torch.empty(0, dtype=dtype, device=self.whole.device)
+
+    def check(self, what="output"):
+        tail = self.whole[self.nbytes:]
+        bad = torch.nonzero(tail != self.fill)
+        assert bad.numel() == 0, "%s: %d guard bytes past the end were written (first at +%d)" % (
+            what, bad.numel(), int(bad[0]))
+
+
+def guarded_outputs(n_chunks, cap=None, device="cuda"):
+    """Guarded fingerprint table, mismatch list (int32 x cap) and count word."""
+    cap = n_chunks if cap is None else cap
+    return Guarded(16 * n_chunks, device), Guarded(4 * cap, device), Guarded(8, device)
+
+
+def fr_diff_guarded(a, b, n_chunks, cap=None):
+    """fr_diff into guarded outputs; returns (ids, count) after checking the guards."""
+    cap = n_chunks if cap is None else cap
+    out, cnt = Guarded(4 * cap), Guarded(8)
+    fr.fr_diff(a, b, n_chunks, out.view(torch.int32) if cap else None, cnt.view(torch.int64))
+    torch.cuda.synchronize()
+    out.check("diff list")
+    cnt.check("diff count")
+    k = int(cnt.view(torch.int64).item())
+    return out.view(torch.int32)[: min(k, cap)], k
+
 
 def host_bytes(tensors):
     return [t.contiguous().view(torch.uint8).cpu().numpy().reshape(-1) for t in tensors]
@@ -61,23 +108,61 @@ def payload_flip_chunks(chunks: np.ndarray, bit_positions: np.ndarray) -> np.nda
     return np.unique(i[ok])
 
 
+def restored_like(tensors, fill=0xA5):
+    """Fresh destination tensors shaped like `tensors`, each at a 256-byte
+    aligned offset of one buffer pre-filled with `fill` and followed by
+    GUARD_BYTES of it.  Returns (tensors, check) where check() asserts that
+    nothing outside the tensors was written."""
+    offs, o = [], 0
+    for t in tensors:
+        offs.append(o)
+        o += (t.numel() * t.element_size() + 255) // 256 * 256 + GUARD_BYTES
+    whole = torch.full((max(o, 1),), fill, dtype=torch.uint8, device="cuda")
+    out = []
+    for t, off in zip(tensors, offs):
+        nb = t.numel() * t.element_size()
+        out.append(whole[off: off + nb].view(t.dtype) if nb else torch.empty(0, dtype=t.dtype, device="cuda"))
+
+    def check():
+        mask = torch.ones(whole.numel(), dtype=torch.bool, device="cuda")
+        for t, off in zip(tensors, offs):
+            mask[off: off + t.numel() * t.element_size()] = False
+        outside = whole[mask]
+        bad = int((outside != fill).sum())
+        assert bad == 0, "%d bytes outside the destination tensors were written" % bad
+
+    return out, check
+
+
 def run_full(tensors, chunk_bytes, flips=None, cap=None):
     """CUDA path over `tensors`: fingerprint, pack, optional flips, unpack into
-    fresh tensors, fingerprint of the restored state.  Returns a dict."""
+    fresh tensors, fingerprint of the restored state, diff.  Every output sits
+    in front of a guard region that is checked after the calls.  Returns a
+    dict."""
     plan = fr.Plan(tensors, chunk_bytes)
-    table = plan.fingerprint()
-    packed = plan.pack()
+    C, P = plan.n_chunks, plan.packed_bytes
+    g_tab, g_pack = Guarded(16 * C), Guarded(P)
+    table = plan.fingerprint(out=g_tab.buf)
+    packed = plan.pack(g_pack.buf)
+    torch.cuda.synchronize()
+    g_tab.check("fingerprint table")
+    g_pack.check("packed buffer")
     if flips is not None and flips.size:
         synth.apply_flips(packed, flips)
-    restored = [torch.full_like(t.view(torch.uint8), 0xA5).view(t.dtype) if t.numel() else torch.empty_like(t)
-                for t in tensors]
+    restored, check_restored = restored_like(tensors)
     plan_r = fr.Plan(restored, chunk_bytes)
-    ids, n = plan_r.unpack_verify(packed, cap=cap)
+    g_tab_r, g_ids, g_cnt = guarded_outputs(C, cap)
+    ids, n = plan_r.unpack_verify(packed, mismatch=g_ids.view(torch.int32), count=g_cnt.view(torch.int64))
     status = plan_r.sync_status()
-    table_r = plan_r.fingerprint()
+    table_r = plan_r.fingerprint(out=g_tab_r.buf)
     torch.cuda.synchronize()
+    g_ids.check("mismatch list")
+    g_cnt.check("mismatch count")
+    g_tab_r.check("restored fingerprint table")
+    check_restored()
+    div, nd = fr_diff_guarded(table, table_r, C)
     out = dict(plan=plan, plan_r=plan_r, table=table, packed=packed, restored=restored, ids=ids, n=n,
-               status=status, table_r=table_r)
+               status=status, table_r=table_r, div=div, nd=nd)
     return out
 
 
@@ -122,6 +207,11 @@ def compare_full(tensors, chunk_bytes, flips=None):
     for i, (g, w) in enumerate(zip(host_bytes(got["restored"]), want["restored"])):
         assert np.array_equal(g, w), "restored tensor %d differs" % i
     assert got["status"] == fr.FR_OK
+    # diff against the oracle's diff of its own two tables
+    want_r = oracle.fingerprint(want["restored"], dtypes, chunk_bytes)
+    ref_div, ref_nd = oracle.diff(want["table"], want_r)
+    assert got["nd"] == ref_nd
+    assert np.array_equal(got["div"].cpu().numpy().astype(np.uint32), ref_div)
     return got, want
 
 

@@ -3,9 +3,10 @@ on the same seeded inputs.
 
 Bar: bit-exact CRC-32C, non-finite counts, packed bytes, mismatch lists and
 restored bytes; sums of squares within 1e-9 relative (exactly equal when the
-sum is zero).  Small workloads are compared whole; the 14-31 GB workloads are
-compared on sampled chunks the oracle computes one by one, plus properties
-that hold at any size.
+sum is zero).  Every workload is compared whole: the small ones through the
+oracle's whole-state calls, the 14-31 GB ones chunk by chunk with the oracle's
+per-chunk calls spread over the host's cores (tests/whole_state.py).  Every
+output buffer is followed by a guard region that must stay untouched.
 """
 import numpy as np
 import pytest
@@ -14,8 +15,9 @@ import torch
 import oracle
 from paper_2509_03047_gb300 import synth
 
-from gpu_helpers import (assert_tables_match, compare_full, expected_mismatch, host_bytes, odd_tensors,
-                         payload_flip_chunks, run_full, table_np)
+from gpu_helpers import (Guarded, assert_tables_match, compare_full, expected_mismatch, fr_diff_guarded,
+                         guarded_outputs, host_bytes, odd_tensors, payload_flip_chunks, table_np)
+from whole_state import WholeState
 
 pytestmark = pytest.mark.gpu
 
@@ -185,7 +187,10 @@ def test_capacity_overflow_and_status():
     synth.apply_flips(packed, np.array(bits))
     restored = [torch.empty_like(t) for t in st]
     pr = fr.Plan(restored, cfg.chunk_bytes)
-    ids, n = pr.unpack_verify(packed, cap=5)
+    _, g_ids, g_cnt = guarded_outputs(C, cap=5)
+    ids, n = pr.unpack_verify(packed, mismatch=g_ids.view(torch.int32), count=g_cnt.view(torch.int64))
+    g_ids.check("mismatch list beyond cap")
+    g_cnt.check("mismatch count")
     assert n == len(bits)
     assert ids.cpu().tolist() == list(range(0, C, 7))[:5]
     assert pr.sync_status() == fr.FR_ERR_CAPACITY
@@ -193,8 +198,9 @@ def test_capacity_overflow_and_status():
     ids, n = pr.unpack_verify(packed)
     assert n == len(bits) and pr.sync_status() == fr.FR_OK
     ta, tb = plan.fingerprint(), pr.fingerprint()
-    d, k = fr.diff(ta, tb, cap=2)
-    assert k == len(bits) and d.cpu().tolist() == list(range(0, C, 7))[:2]
+    for cap in (0, 1, 2):
+        d, k = fr_diff_guarded(ta, tb, C, cap=cap)
+        assert k == len(bits) and d.cpu().tolist() == list(range(0, C, 7))[:cap]
 
 
 def test_argument_errors():
@@ -250,123 +256,107 @@ def test_pinned_host_transfer_buffer():
 
 # ------------------------------------------------------------------ full-size workloads
 
-def _sample_chunks(C, k, seed):
-    rng = np.random.default_rng(seed)
-    picks = set(rng.choice(C, size=min(k, C), replace=False).tolist()) | {0, C - 1}
-    return sorted(picks)
-
-
-def _check_sampled(state, chunk_bytes, table, packed, sample):
-    """Per sampled chunk: the oracle's fingerprint of its bytes, its header and
-    its payload + padding in the packed buffer."""
-    tab = table_np(table)
-    nbytes = [t.numel() * t.element_size() for t in state]
-    dts = [fr.fr_dtype_of(t) for t in state]
-    chunks, packed_bytes = oracle.plan(nbytes, dts, chunk_bytes)
-    assert packed.numel() == packed_bytes
-    raw = [t.view(torch.uint8) for t in state]
-    for c in sample:
-        ch = chunks[c]
-        t, off, ln, poff = int(ch["tensor_idx"]), int(ch["tensor_off"]), int(ch["len"]), int(ch["payload_off"])
-        data = raw[t][off:off + ln].cpu().numpy()
-        crc, nf, s = oracle.fingerprint_chunk(data, dts[t])
-        got = tab[c]
-        assert int(got["crc32c"]) == crc and int(got["nonfinite"]) == nf, c
-        assert (s == 0 and got["sumsq"] == 0) or abs(got["sumsq"] - s) <= 1e-9 * abs(s), c
-        hdr = packed[64 * c: 64 * c + 64].cpu().numpy().tobytes()
-        assert hdr == oracle.header(ch, c, (crc, nf, s if s == got["sumsq"] else float(got["sumsq"]))), c
-        assert torch.equal(packed[poff:poff + ln], raw[t][off:off + ln]), c
-        pad_end = poff + (ln + 255) // 256 * 256
-        assert int(packed[poff + ln:pad_end].count_nonzero()) == 0, c
-    return chunks
-
-
-def _big_config(name, sample_k=48):
+def _whole_config(name):
+    """A full-size workload through the C ABI, every chunk compared with the
+    oracle (tests/whole_state.py): fingerprint table, packed headers, payloads
+    and padding; then the config's bit flips, unpack_verify into fresh
+    tensors, and the mismatch list, restored bytes, restored table and diff.
+    Every output buffer has a guard region checked after its call."""
     cfg = synth.get_config(name)
     st = synth.make_state(cfg, "cuda")
     pos = synth.inject_nonfinite(cfg, st)
     plan = fr.Plan(st, cfg.chunk_bytes)
-    table = plan.fingerprint()
-    packed = plan.pack()
+    C, P = plan.n_chunks, plan.packed_bytes
+    g_tab, g_pack = Guarded(16 * C), Guarded(P)
+    table = plan.fingerprint(out=g_tab.buf)
+    packed = plan.pack(g_pack.buf)
     torch.cuda.synchronize()
-    sample = _sample_chunks(plan.n_chunks, sample_k, 7)
-    chunks = _check_sampled(st, cfg.chunk_bytes, table, packed, sample)
-    # any-size properties
+    g_tab.check("fingerprint table")
+    g_pack.check("packed buffer")
+    ws = WholeState(st, [fr.fr_dtype_of(t) for t in st], cfg.chunk_bytes)
+    assert ws.C == C and ws.packed_bytes == P
     tab = table_np(table)
+    fails = ws.check_pack(tab, packed)
+    assert not fails, "%d chunk checks failed, first %s" % (len(fails), fails[:5])
     assert int(tab["nonfinite"].sum()) == pos.size
-    assert int(packed[64 * plan.n_chunks: int(chunks["payload_off"][0])].count_nonzero()) == 0
-    return cfg, st, pos, plan, table, packed, chunks
 
-
-def _restore_with_flips(cfg, st, plan, table, packed, chunks):
-    flips = synth.flip_positions(plan.packed_bytes, cfg.flips, cfg.seed)
+    flips = synth.flip_positions(P, cfg.flips, cfg.seed)
     synth.apply_flips(packed, flips)
     restored = [torch.empty_like(t) for t in st]
     pr = fr.Plan(restored, cfg.chunk_bytes)
-    ids, n = pr.unpack_verify(packed)
+    g_tab_r, g_ids, g_cnt = guarded_outputs(C)
+    ids, n = pr.unpack_verify(packed, mismatch=g_ids.view(torch.int32), count=g_cnt.view(torch.int64))
     assert pr.sync_status() == fr.FR_OK
-    want = expected_mismatch(chunks, flips)
-    assert np.array_equal(ids.cpu().numpy().astype(np.int64), want)
-    # restored bytes are the packed payload bytes: they differ from the
-    # original in exactly the flipped payload bits
-    pay = payload_flip_chunks(chunks, flips)
-    diffbits = 0
-    for a, b in zip(st, restored):
-        x = torch.bitwise_xor(a.view(torch.uint8), b.view(torch.uint8))
-        diffbits += int(sum(bin(i).count("1") * int(c) for i, c in
-                            enumerate(torch.bincount(x.view(-1).to(torch.int64), minlength=256).tolist()) if i))
-    b = flips // 8
-    starts = chunks["payload_off"].astype(np.int64)
-    i = np.clip(np.searchsorted(starts, b, side="right") - 1, 0, None)
-    in_payload = (b >= starts[0]) & (b < starts[i] + chunks["len"][i].astype(np.int64))
-    assert diffbits == int(in_payload.sum())
-    tr = pr.fingerprint()
-    d, k = fr.diff(table, tr)
-    assert np.array_equal(d.cpu().numpy().astype(np.int64), pay)
-    return pr, restored
+    table_r = pr.fingerprint(out=g_tab_r.buf)
+    torch.cuda.synchronize()
+    for g, what in ((g_ids, "mismatch list"), (g_cnt, "mismatch count"), (g_tab_r, "restored table")):
+        g.check(what)
+    fails, want_ids = ws.check_restore(packed, restored, table_np(table_r))
+    assert not fails, "%d restore checks failed, first %s" % (len(fails), fails[:5])
+    got_ids = ids.cpu().numpy().astype(np.uint32)
+    assert n == want_ids.size and np.array_equal(got_ids, want_ids)
+    # and where the flips landed, from the documented layout alone
+    assert np.array_equal(got_ids.astype(np.int64), expected_mismatch(ws.chunks, flips))
+    div, nd = fr_diff_guarded(table, table_r, C)
+    want_div, want_nd = ws.oracle_diff()
+    assert nd == want_nd and np.array_equal(div.cpu().numpy().astype(np.uint32), want_div)
+    assert np.array_equal(want_div.astype(np.int64), payload_flip_chunks(ws.chunks, flips))
+    print("%s: %d chunks, oracle passes %.1f s + %.1f s on %d threads, %d mismatching, %d diverged" % (
+        name, C, ws.seconds["pack_pass"], ws.seconds["restore_pass"], ws.threads, n, nd))
+    return cfg, st, plan, table, ws
 
 
-def test_l8b_tp8_full_size_sampled():
-    cfg, st, pos, plan, table, packed, chunks = _big_config("l8b_tp8")
+def test_l8b_tp8_whole_state():
+    cfg, st, plan, table, ws = _whole_config("l8b_tp8")
     assert plan.n_chunks == 3806
-    _restore_with_flips(cfg, st, plan, table, packed, chunks)
 
 
-def test_l70b_tp8pp4_full_size_sampled():
-    cfg, st, pos, plan, table, packed, chunks = _big_config("l70b_tp8pp4", sample_k=40)
-    assert plan.n_chunks == 2212 and pos.size == 50
-    _restore_with_flips(cfg, st, plan, table, packed, chunks)
+def test_l70b_tp8pp4_whole_state():
+    cfg, st, plan, table, ws = _whole_config("l70b_tp8pp4")
+    assert plan.n_chunks == 2212
 
 
-def test_l70b_pinned_host_variant_sampled():
+def test_l70b_pinned_host_variant():
+    """The first 10 parameter tensors of the 70B shard packed into pinned host
+    memory: the same bytes as the device pack (itself checked against the
+    oracle above), guard intact, and a clean restore from the host buffer."""
     cfg = synth.get_config("l70b_tp8pp4")
-    st = synth.make_state(cfg, "cuda")[:40]  # the first 10 parameter tensors
+    st = synth.make_state(cfg, "cuda")[:40]
     plan = fr.Plan(st, cfg.chunk_bytes)
     dev = plan.pack()
-    host = plan.new_packed(pinned=True)
-    plan.pack(host)
+    host = Guarded(plan.packed_bytes, pinned=True)
+    plan.pack(host.buf)
     torch.cuda.synchronize()
-    assert torch.equal(dev.cpu(), host)
+    host.check("pinned packed buffer")
+    assert torch.equal(dev.cpu(), host.buf)
     restored = [torch.empty_like(t) for t in st]
     pr = fr.Plan(restored, cfg.chunk_bytes)
-    ids, n = pr.unpack_verify(host)
+    ids, n = pr.unpack_verify(host.buf)
     assert n == 0
     assert all(torch.equal(a.view(torch.uint8), b.view(torch.uint8)) for a, b in zip(st, restored))
 
 
-def test_zero_frag_full_size_sampled_and_diff():
-    cfg, st, pos, plan, table, packed, chunks = _big_config("zero_frag", sample_k=64)
-    assert plan.n_chunks == len(chunks) and pos.size > 0
-    del packed
-    torch.cuda.empty_cache()
-    rows = [(int(c["tensor_idx"]), int(c["tensor_off"]), int(c["len"]), int(c["dtype"])) for c in chunks]
+def test_zero_frag_whole_state_and_diff():
+    cfg, st, plan, table, ws = _whole_config("zero_frag")
+    assert ws.C == 132976
+    rows = [(int(c["tensor_idx"]), int(c["tensor_off"]), int(c["len"]), int(c["dtype"])) for c in ws.chunks]
     mod = [t.clone() for t in st]
     ids = synth.modify_for_diff(cfg, mod, rows)
     pm = fr.Plan(mod, cfg.chunk_bytes)
     tm = pm.fingerprint()
-    d, k = fr.diff(table, tm)
+    d, k = fr_diff_guarded(table, tm, plan.n_chunks)
     assert k == cfg.diff_chunks == 100
     assert np.array_equal(d.cpu().numpy().astype(np.int64), ids)
+    # the oracle on the modified chunks: exactly these entries change
+    want_m = ws.table.copy()
+    raw = [t.view(torch.uint8) for t in mod]
+    for c in ids.tolist():
+        ch = ws.chunks[c]
+        t, off, ln = int(ch["tensor_idx"]), int(ch["tensor_off"]), int(ch["len"])
+        want_m[c] = oracle.fingerprint_chunk(raw[t][off:off + ln].cpu().numpy(), int(ch["dtype"]))
+    assert_tables_match(table_np(tm)[ids], want_m[ids], "modified chunks")
+    od, on = oracle.diff(ws.table, want_m)
+    assert on == 100 and np.array_equal(od.astype(np.int64), ids)
 
 
 def test_chunk_larger_than_4_gib():

@@ -13,7 +13,7 @@ import torch
 
 from paper_2509_03047_gb300 import synth
 
-from gpu_helpers import assert_tables_match, odd_tensors, table_np
+from gpu_helpers import Guarded, assert_tables_match, odd_tensors, table_np
 
 pytestmark = pytest.mark.gpu
 
@@ -22,10 +22,11 @@ fr = pytest.importorskip("paper_2509_03047_gb300.flashrec")
 
 def _static_table(tensors, chunk):
     n = fr.Plan(tensors, chunk).n_chunks
-    out = torch.full((n * 16,), 0xEE, dtype=torch.uint8, device="cuda")
-    fr.fr_fingerprint_static(tensors, chunk, out)
+    out = Guarded(n * 16)
+    fr.fr_fingerprint_static(tensors, chunk, out.buf)
     torch.cuda.synchronize()
-    return out
+    out.check("static fingerprint table")
+    return out.buf
 
 
 def test_static_entry_point_matches_plan_on_three_calls_in_a_row():
@@ -52,6 +53,7 @@ def test_static_entry_point_rejects_inputs_beyond_its_limit():
     with pytest.raises(fr.FlashrecError) as e:
         fr.fr_fingerprint_static([t], 4, out)
     assert e.value.status == fr.FR_ERR_INVALID_ARG
+    assert "FR_STATIC_MAX_CHUNKS" in fr.fr_last_error()
     # the largest allowed input still works
     ok = t[: 4 * fr.FR_STATIC_MAX_CHUNKS]
     got = _static_table([ok], 4)
