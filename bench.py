@@ -20,6 +20,7 @@ Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl flashrec|refe
 from __future__ import annotations
 
 import argparse
+import gc
 import json
 import os
 import statistics
@@ -240,7 +241,9 @@ def run_flashrec(args):
     stream = torch.cuda.current_stream()
     n_cls = sweep_classes(src)
 
-    def step(ev=None, buf=packed, sync_counts=False):
+    def step(ev=None, buf=None, sync_counts=False):
+        if buf is None:
+            buf = packed
         if ev:
             ev[0].record(stream)
         fr.fr_fingerprint(plan_s.handle, tab_s, stream)
@@ -526,7 +529,8 @@ def run_flashrec(args):
     if ws == 1 and args.workloads:
         plan_s.close()
         plan_d.close()
-        del src, dst, packed, tab_s, tab_d, plan_s, plan_d
+        del src, dst, packed, tab_s, tab_d, plan_s, plan_d, step, fused_step
+        gc.collect()
         torch.cuda.synchronize()
         torch.cuda.empty_cache()
         held = torch.cuda.memory_allocated(dev)
