@@ -15,9 +15,11 @@
 //    own bank, so the 32 lookups of a warp never conflict.  At the end of a
 //    piece the streams are folded with GF(2) multiplications by constants and
 //    warp shuffles into the raw CRC of the piece;
-//  * non-finite count and sum of squares, fused on the same registers: exact
-//    squares (fp32: x*x and fma(x,x,-x*x); bf16: x*x is already exact) summed
-//    with error-free TwoSum in packed f32x2 arithmetic, flushed into fp64.  A
+//  * non-finite count and sum of squares, fused on the same registers: each
+//    square is added to a packed f32x2 running sum by one FMA, and the
+//    addition's error -- including the square's own rounding for fp32 -- is
+//    recovered to second order by a TwoSum whose low term is a second FMA
+//    (two_sum_sq), then flushed into fp64.  A
 //    stage whose running sum is not finite (NaN/Inf input, or overflow) or is
 //    tiny with non-zero input is discarded and redone element by element in
 //    fp64 from a reload of its 16-byte units, so the fast path never needs a
@@ -228,10 +230,32 @@ __device__ __forceinline__ u64 sub2(u64 a, u64 b) {
   asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
   return r;
 }
-__device__ __forceinline__ u64 mul2(u64 a, u64 b) {
+
+__device__ __forceinline__ u64 fma2(u64 a, u64 b, u64 c) {
   u64 r;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
   return r;
+}
+
+// S + C += x*x, for each half of a packed pair (S, x >= 0 in effect: squares
+// and sums of squares).  t = fl(S + x*x) by one FMA; then zn = fl(S - t),
+// y = t + zn, a = S - y, b = fl(x*x + zn) by a second FMA, and C takes a + b.
+//  * t <= 2S: S - t is exact (Sterbenz), so zn = S - t, y = S, a = 0 and b is
+//    the addition's exact error S + x*x - t rounded once.
+//  * t > 2S: zn lies in [-t, -t/2], so y = t + zn is exact and equals S + d,
+//    d the rounding error of S - t; a = -d exactly, and b = (error + d)
+//    rounded once, with |error + d| <= ulp(t).
+// Either way a + b is the error of t to within about 3u^2 t (u = 2^-24): the
+// square need not be exact in fp32, so fp32 inputs need no separate residual
+// term, and for bf16 inputs (exact squares) this is Knuth's TwoSum exactly.
+__device__ __forceinline__ void two_sum_sq(u64& S, u64& C, u64 x) {
+  const u64 t = fma2(x, x, S);
+  const u64 zn = sub2(S, t);
+  const u64 y = add2(t, zn);
+  const u64 a = sub2(S, y);
+  const u64 b = fma2(x, x, zn);
+  C = add2(C, add2(a, b));
+  S = t;
 }
 
 // S + C += p, error-free (Knuth's TwoSum): S takes the rounded sum, C the
@@ -253,25 +277,16 @@ struct FpAcc {
 template <int DT>
 __device__ __forceinline__ void fp_unit(const uint4& v, FpAcc& f) {
   if (DT == kDtF32) {
-    const u64 x01 = pk(v.x, v.y), x23 = pk(v.z, v.w);
-    const u64 p01 = mul2(x01, x01), p23 = mul2(x23, x23);
-    // x*x = p + e exactly (fp32 product, FMA residual)
-    const float e0 = __fmaf_rn(__uint_as_float(v.x), __uint_as_float(v.x), -lo_f(p01));
-    const float e1 = __fmaf_rn(__uint_as_float(v.y), __uint_as_float(v.y), -hi_f(p01));
-    const float e2 = __fmaf_rn(__uint_as_float(v.z), __uint_as_float(v.z), -lo_f(p23));
-    const float e3 = __fmaf_rn(__uint_as_float(v.w), __uint_as_float(v.w), -hi_f(p23));
-    two_sum_acc(f.A, f.CA, p01);
-    f.CA = add2(f.CA, pk(__float_as_uint(e0), __float_as_uint(e1)));
-    two_sum_acc(f.B, f.CB, p23);
-    f.CB = add2(f.CB, pk(__float_as_uint(e2), __float_as_uint(e3)));
+    two_sum_sq(f.A, f.CA, pk(v.x, v.y));
+    two_sum_sq(f.B, f.CB, pk(v.z, v.w));
   } else {
     // bf16 pairs: the low element is the low half-word
     const u64 y0 = pk(v.x << 16, v.x & 0xFFFF0000u), y1 = pk(v.y << 16, v.y & 0xFFFF0000u);
     const u64 y2 = pk(v.z << 16, v.z & 0xFFFF0000u), y3 = pk(v.w << 16, v.w & 0xFFFF0000u);
-    two_sum_acc(f.A, f.CA, mul2(y0, y0));
-    two_sum_acc(f.B, f.CB, mul2(y2, y2));
-    two_sum_acc(f.A, f.CA, mul2(y1, y1));
-    two_sum_acc(f.B, f.CB, mul2(y3, y3));
+    two_sum_sq(f.A, f.CA, y0);
+    two_sum_sq(f.B, f.CB, y2);
+    two_sum_sq(f.A, f.CA, y1);
+    two_sum_sq(f.B, f.CB, y3);
   }
 }
 
