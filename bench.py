@@ -512,7 +512,9 @@ def run_flashrec(args):
                         "frac_median": round((P / med_e2e) / (half / statistics.median(t_links)), 4),
                         "how": "cudaMemcpyAsync of P/2 bytes device->host and P/2 host->device at once, 64 MiB "
                                "pieces on two streams, pinned host memory, best and median of 5; the restore "
-                               "moves P each way"},
+                               "moves P each way with the sweep kernels' own loads and stores over the same "
+                               "link, which is not bound to the copy engines' rate (frac > 1 when they are "
+                               "slower)"},
                "serial": {"value": round(sum_over_ranks(SWEEPS_PER_STEP * S / t_serial / 1e9, dev), 2),
                           "ms_per_step": ms(t_serial), "ms_median": ms(med_serial), "ms_best": ms(best_serial),
                           "how": "fr_pack to the host buffer, then fr_unpack_verify from it, with the flips"}}

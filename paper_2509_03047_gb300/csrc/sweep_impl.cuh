@@ -361,6 +361,14 @@ __device__ __forceinline__ void prefetch_l2(const uint8_t* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
+// The same, issued by lane 0 only, as a predicated instruction (no branch).
+__device__ __forceinline__ void prefetch_l2_lane0(const uint8_t* p, uint32_t bytes, uint32_t lane) {
+  asm volatile(
+      "{\n\t.reg .pred q;\n\tsetp.eq.u32 q, %2, 0;\n\t@q cp.async.bulk.prefetch.L2.global [%0], %1;\n\t}" ::"l"(p),
+      "r"(bytes), "r"(lane)
+      : "memory");
+}
+
 // Per-mode pipeline geometry: blocks per lane held in registers one stage
 // ahead, and spans (kSpan blocks) prefetched into L2 ahead of use.
 template <int MODE>
@@ -462,9 +470,10 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
   const uint8_t* sp = src + lane * 16;
   uint8_t* wp = dst + lane * 16;
 
-  if (kAhead > 0 && SAL == 16 && lane == 0) {
-    const uint64_t first = nblk < kSpan * kAhead ? nblk : kSpan * kAhead;
-    prefetch_l2(src, static_cast<uint32_t>(first * kBlockBytes));
+  // The first span goes to L2 now; each later one about a span before use.
+  if (kAhead > 0 && SAL == 16) {
+    const uint64_t n = nblk < kSpan ? nblk : kSpan;
+    prefetch_l2_lane0(src, static_cast<uint32_t>(n * kBlockBytes), lane);
   }
 
   Lane<MODE, DT> L;
@@ -478,10 +487,17 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
     if (u < nblk) cur[u] = ld_unit<SAL>(sp + static_cast<uint64_t>(u) * kBlockBytes);
   const uint8_t* lp = sp + kStageBytes;  // the next stage's loads
 
-  uint64_t i = 0;
-  // Steady state: whole spans whose following stage is whole too.  The inner
-  // stage loop has no branch at all; the span's prefetch and validity check
-  // sit outside it.
+  // Three loops cover a piece: (1) whole spans whose following stage is
+  // whole too, each span (one sum segment) a call-free loop of kSpan/kStage
+  // stages with no branch, preceded by the L2 prefetch of the span kAhead
+  // ahead and followed by its validity check -- the bulk of a long piece;
+  // (2) the stages left whose following stage is still whole, one stage per
+  // iteration, a span's check and the next prefetch when a stage ends a span;
+  // (3) the last one or two stages, predicated.  Loop (2) keeps the
+  // predicated drain to under 2 * kStage blocks (it used to take the last
+  // span and a stage, and ran at half speed); loop (1) keeps long pieces on
+  // the tighter loop (with (2) alone the bf16 fingerprint lost 12% per warp).
+  uint64_t i = 0;  // first block of the current span
   for (; i + kSpan + kStage <= nblk; i += kSpan) {
     if (kAhead > 0 && SAL == 16 && lane == 0) {
       const uint64_t pf = i + kSpan * kAhead;
@@ -491,7 +507,7 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
       }
     }
 #pragma unroll 1
-    for (int st = 0; st < kSpan / kStage; ++st) {
+    for (int stg = 0; stg < kSpan / kStage; ++stg) {
 #pragma unroll
       for (int u = 0; u < kStage; ++u) {
         if (Geo<MODE>::kLoadFirst) {
@@ -508,7 +524,48 @@ __device__ __forceinline__ void sweep_piece(const uint8_t* __restrict__ src, uin
     }
     if (kFp) span_end<MODE, DT, SAL>(L, sp, i, i + kSpan, segs + i / kSpan, lane);
   }
-  // Drain: the last (partial) span and the stage after it, with predicates.
+  if (kAhead > 0 && SAL == 16) {  // loop (2) prefetches at span ends only
+    const uint64_t pf = i + kSpan * kAhead;
+    if (pf < nblk) {
+      const uint64_t n = (nblk - pf < kSpan) ? nblk - pf : kSpan;
+      prefetch_l2_lane0(src + pf * kBlockBytes, static_cast<uint32_t>(n * kBlockBytes), lane);
+    }
+  }
+  // Loop (2): stage j after i is steady if i + (j + 2) * kStage <= nblk.
+  uint32_t st = 0;  // stages of the current span done
+  const uint64_t left = nblk - i;
+  const uint32_t n_steady = left >= 2 * kStage ? static_cast<uint32_t>((left - kStage) / kStage) : 0u;
+#pragma unroll 1
+  for (uint32_t k = n_steady; k > 0; --k) {
+#pragma unroll
+    for (int u = 0; u < kStage; ++u) {
+      if (Geo<MODE>::kLoadFirst) {
+        const uint4 v = cur[u];
+        cur[u] = ld_unit<SAL>(lp + u * kBlockBytes);
+        do_unit<MODE, DT, DAL>(L, v, wp + u * kBlockBytes, lb);
+      } else {
+        do_unit<MODE, DT, DAL>(L, cur[u], wp + u * kBlockBytes, lb);
+        cur[u] = ld_unit<SAL>(lp + u * kBlockBytes);
+      }
+    }
+    lp += kStageBytes;
+    wp += kStageBytes;
+    if (++st == kSpan / kStage) {
+      st = 0;
+      if (kFp) span_end<MODE, DT, SAL>(L, sp, i, i + kSpan, segs + i / kSpan, lane);
+      if (kAhead > 0 && SAL == 16) {
+        const uint64_t pf = i + kSpan + kSpan * kAhead;
+        if (pf < nblk) {
+          const uint64_t n = (nblk - pf < kSpan) ? nblk - pf : kSpan;
+          prefetch_l2_lane0(src + pf * kBlockBytes, static_cast<uint32_t>(n * kBlockBytes), lane);
+        }
+      }
+      i += kSpan;
+    }
+  }
+  i += static_cast<uint64_t>(st) * kStage;
+  // Drain: the last one or two stages (fewer than 2 * kStage blocks), with
+  // predicates.
   for (; i < nblk; i += kStage) {
 #pragma unroll
     for (int u = 0; u < kStage; ++u) {
