@@ -12,6 +12,7 @@
 // kernels only overlap on disjoint SMs).  All device memory and events a plan
 // needs are created here, at creation; the sweep calls only launch kernels.
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <cstdarg>
@@ -113,6 +114,16 @@ fr_status invalid(const char* what) {
   set_err("invalid argument: %s", what);
   return FR_ERR_INVALID_ARG;
 }
+
+// A named NVTX range around each public call, so a profiler's timeline shows
+// which call issued which kernels.  NVTX is header-only: with no profiler
+// attached, push and pop return at once.
+struct CallRange {
+  explicit CallRange(const char* name) { nvtxRangePushA(name); }
+  ~CallRange() { nvtxRangePop(); }
+  CallRange(const CallRange&) = delete;
+  CallRange& operator=(const CallRange&) = delete;
+};
 
 fr_status cuda_fail(cudaError_t e, const char* where) {
   set_err("%s: %s", where, cudaGetErrorString(e));
@@ -510,6 +521,7 @@ int fr_version(void) { return 10100; }
 
 fr_status fr_plan_create_batched(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes,
                                  uint32_t n_batches, fr_plan* out) {
+  CallRange nvtx("fr_plan_create_batched");
   if (out == nullptr) return invalid("out is null");
   *out = nullptr;
   if (n_tensors > 0 && tensors == nullptr) return invalid("tensors is null");
@@ -675,6 +687,7 @@ fr_status fr_plan_batch(fr_plan p, uint32_t batch, uint32_t* n_batches, uint64_t
 }
 
 void fr_plan_destroy(fr_plan p) {
+  CallRange nvtx("fr_plan_destroy");
   if (p == nullptr) return;
   DeviceGuard g(p->device);
   cudaDeviceSynchronize();
@@ -683,6 +696,7 @@ void fr_plan_destroy(fr_plan p) {
 }
 
 fr_status fr_fingerprint(fr_plan p, fr_fp* out_dev, void* stream) {
+  CallRange nvtx("fr_fingerprint");
   if (p == nullptr) return invalid("plan is null");
   if (p->n_chunks == 0) return FR_OK;
   if (out_dev == nullptr) return invalid("out_dev is null");
@@ -693,10 +707,12 @@ fr_status fr_fingerprint(fr_plan p, fr_fp* out_dev, void* stream) {
 }
 
 fr_status fr_pack(fr_plan p, void* dst, uint64_t dst_bytes, void* stream) {
+  CallRange nvtx("fr_pack");
   return fr_pack_fp(p, dst, dst_bytes, nullptr, stream);
 }
 
 fr_status fr_pack_fp(fr_plan p, void* dst, uint64_t dst_bytes, fr_fp* fp_dev, void* stream) {
+  CallRange nvtx("fr_pack_fp");
   if (p == nullptr) return invalid("plan is null");
   if (p->n_chunks == 0) return FR_OK;
   fr_status st = check_packed_buffer(p, dst, dst_bytes);
@@ -709,11 +725,13 @@ fr_status fr_pack_fp(fr_plan p, void* dst, uint64_t dst_bytes, fr_fp* fp_dev, vo
 
 fr_status fr_unpack_verify(fr_plan p, const void* src, uint64_t src_bytes, uint32_t* mismatch_dev, uint64_t cap,
                            uint64_t* n_mismatch_dev, void* stream) {
+  CallRange nvtx("fr_unpack_verify");
   return fr_unpack_verify_fp(p, src, src_bytes, mismatch_dev, cap, n_mismatch_dev, nullptr, stream);
 }
 
 fr_status fr_unpack_verify_fp(fr_plan p, const void* src, uint64_t src_bytes, uint32_t* mismatch_dev, uint64_t cap,
                               uint64_t* n_mismatch_dev, fr_fp* fp_dev, void* stream) {
+  CallRange nvtx("fr_unpack_verify_fp");
   if (p == nullptr) return invalid("plan is null");
   if (n_mismatch_dev == nullptr) return invalid("n_mismatch_dev is null");
   if (cap > 0 && mismatch_dev == nullptr) return invalid("mismatch_dev is null");
@@ -735,6 +753,7 @@ fr_status fr_unpack_verify_fp(fr_plan p, const void* src, uint64_t src_bytes, ui
 }
 
 fr_status fr_pack_batch(fr_plan p, uint32_t batch, void* dst, uint64_t dst_bytes, void* stream) {
+  CallRange nvtx("fr_pack_batch");
   if (p == nullptr) return invalid("plan is null");
   if (p->n_chunks == 0) return FR_OK;
   if (batch >= p->n_batches) return invalid("batch out of range");
@@ -747,6 +766,7 @@ fr_status fr_pack_batch(fr_plan p, uint32_t batch, void* dst, uint64_t dst_bytes
 }
 
 fr_status fr_unpack_verify_batch(fr_plan p, uint32_t batch, const void* src, uint64_t src_bytes, void* stream) {
+  CallRange nvtx("fr_unpack_verify_batch");
   if (p == nullptr) return invalid("plan is null");
   if (p->n_chunks == 0) return FR_OK;
   if (batch >= p->n_batches) return invalid("batch out of range");
@@ -760,6 +780,7 @@ fr_status fr_unpack_verify_batch(fr_plan p, uint32_t batch, const void* src, uin
 
 fr_status fr_unpack_collect(fr_plan p, uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev,
                             void* stream) {
+  CallRange nvtx("fr_unpack_collect");
   if (p == nullptr) return invalid("plan is null");
   if (n_mismatch_dev == nullptr) return invalid("n_mismatch_dev is null");
   if (cap > 0 && mismatch_dev == nullptr) return invalid("mismatch_dev is null");
@@ -777,6 +798,7 @@ fr_status fr_unpack_collect(fr_plan p, uint32_t* mismatch_dev, uint64_t cap, uin
 fr_status fr_restore(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint32_t max_retries,
                      uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev, void* stream_src,
                      void* stream_dst) {
+  CallRange nvtx("fr_restore");
   return fr_restore_fp(src, dst, staging, staging_bytes, max_retries, mismatch_dev, cap, n_mismatch_dev, nullptr,
                        nullptr, stream_src, stream_dst);
 }
@@ -784,6 +806,7 @@ fr_status fr_restore(fr_plan src, fr_plan dst, void* staging, uint64_t staging_b
 fr_status fr_restore_fp(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint32_t max_retries,
                         uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev, fr_fp* fp_src_dev,
                         fr_fp* fp_dst_dev, void* stream_src, void* stream_dst) {
+  CallRange nvtx("fr_restore_fp");
   if (src == nullptr || dst == nullptr) return invalid("plan is null");
   if (n_mismatch_dev == nullptr) return invalid("n_mismatch_dev is null");
   if (cap > 0 && mismatch_dev == nullptr) return invalid("mismatch_dev is null");
@@ -833,6 +856,7 @@ fr_status fr_restore_fp(fr_plan src, fr_plan dst, void* staging, uint64_t stagin
 fr_status fr_restore_multi(const fr_plan* src, uint32_t n_src, fr_plan dst, void* staging, uint64_t staging_bytes,
                            uint32_t max_retries, uint32_t* mismatch_dev, uint64_t cap, uint64_t* n_mismatch_dev,
                            fr_fp* fp_dst_dev, void* const* streams_src, void* stream_dst) {
+  CallRange nvtx("fr_restore_multi");
   if (src == nullptr || n_src == 0) return invalid("no source plans");
   if (dst == nullptr) return invalid("plan is null");
   if (n_mismatch_dev == nullptr) return invalid("n_mismatch_dev is null");
@@ -890,11 +914,13 @@ fr_status fr_restore_multi(const fr_plan* src, uint32_t n_src, fr_plan dst, void
 
 fr_status fr_resend(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint64_t* n_resent,
                     void* stream_src, void* stream_dst) {
+  CallRange nvtx("fr_resend");
   return fr_resend_fp(src, dst, staging, staging_bytes, n_resent, nullptr, nullptr, stream_src, stream_dst);
 }
 
 fr_status fr_resend_fp(fr_plan src, fr_plan dst, void* staging, uint64_t staging_bytes, uint64_t* n_resent,
                        fr_fp* fp_src_dev, fr_fp* fp_dst_dev, void* stream_src, void* stream_dst) {
+  CallRange nvtx("fr_resend_fp");
   if (src == nullptr || dst == nullptr) return invalid("plan is null");
   fr_status st = check_same_layout(src, dst);
   if (st != FR_OK) return st;
@@ -914,6 +940,7 @@ fr_status fr_resend_fp(fr_plan src, fr_plan dst, void* staging, uint64_t staging
 
 fr_status fr_diff(const fr_fp* a_dev, const fr_fp* b_dev, uint64_t n_chunks, uint32_t* diverged_dev, uint64_t cap,
                   uint64_t* n_out_dev, void* stream) {
+  CallRange nvtx("fr_diff");
   if (n_out_dev == nullptr) return invalid("n_out_dev is null");
   if (cap > 0 && diverged_dev == nullptr) return invalid("diverged_dev is null");
   if (n_chunks >= (1ull << 32)) return invalid("too many chunks");
@@ -931,6 +958,7 @@ fr_status fr_diff(const fr_fp* a_dev, const fr_fp* b_dev, uint64_t n_chunks, uin
 }
 
 fr_status fr_sync_status(fr_plan p, void* stream) {
+  CallRange nvtx("fr_sync_status");
   if (p == nullptr) return invalid("plan is null");
   DeviceGuard g(p->device);
   if (!g.ok) return cuda_fail(cudaGetLastError(), "select plan device");
