@@ -40,6 +40,16 @@ using namespace frk;
 #ifndef FR_MIX_PACK
 #define FR_MIX_PACK 1
 #endif
+// Pack and unpack launches keep this percentage of each class's segments out
+// of the warps' own ranges and cut it into units of FR_UNIT_SEGS_PACK
+// segments, which warps claim at run time once their range is done (0: none;
+// the fingerprint keeps a static split).
+#ifndef FR_DYN_PCT_PACK
+#define FR_DYN_PCT_PACK 8
+#endif
+#ifndef FR_UNIT_SEGS_PACK
+#define FR_UNIT_SEGS_PACK 4
+#endif
 
 
 namespace {
@@ -52,6 +62,10 @@ struct SweepClass {
   bool aligned = false;
   uint64_t warp_off = 0;
   uint64_t list_off = 0;
+  // mixed: per sweep class, its claimable units and where its chunk list starts
+  uint32_t unit_off[kClassCount] = {0, 0, 0, 0, 0, 0};
+  uint32_t n_units[kClassCount] = {0, 0, 0, 0, 0, 0};
+  uint32_t class_list[kClassCount] = {0, 0, 0, 0, 0, 0};
 };
 
 struct BatchInfo {
@@ -73,7 +87,14 @@ struct Decomp {
   uint64_t* d_rec_nblk = nullptr;
   uint32_t* d_rec_mul = nullptr;  // per record: x^(8 * bytes after it in its chunk's body)
   Record* d_recs = nullptr;
+  WarpDesc* d_units = nullptr;  // mixed: claimable units of every batch
+  uint32_t* d_queue = nullptr;  // mixed: kQueueWords counters per batch (SweepParams::queue)
 };
+
+// Counters of one mixed launch: a claim count per class and a count of the
+// warps that have left (kernels.h, SweepParams::queue), padded to 32 bytes.
+constexpr size_t kQueueWords = 8;
+static_assert(kQueueWords >= kClassCount + 1, "queue words");
 
 }  // namespace
 
@@ -197,6 +218,8 @@ void free_decomp(Decomp& D) {
   cudaFree(D.d_rec_nblk);
   cudaFree(D.d_rec_mul);
   cudaFree(D.d_recs);
+  cudaFree(D.d_units);
+  cudaFree(D.d_queue);
   D = Decomp();
 }
 
@@ -221,7 +244,11 @@ void free_device(fr_plan p) {
 // to allocate at least (list-mode calls use one slot per listed chunk).
 // Plain: every class gets all n_ctas * warps_per_cta warps (one launch per
 // class).  Mixed: the classes of a batch share them in proportion to their
-// weighted blocks, each class's warps spread round-robin over the CTAs.
+// weighted blocks, each class's warps spread round-robin over the CTAs.  For
+// pack and unpack (mix 2) the warps' ranges cover the first
+// (100 - FR_DYN_PCT_PACK)% of each class's segments and the rest becomes units
+// claimed at run time (their records follow the class's range records, in
+// block order).
 cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<uint64_t>& bounds, int n_ctas,
                          int warps_per_cta, int mix, uint64_t min_recs, Decomp& D) {
   const bool mixed = mix != 0;  // 1: fingerprint weights, 2: pack / unpack weights
@@ -234,6 +261,10 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
   std::vector<uint32_t> lists;
   std::vector<uint64_t> rec_nblk;
   std::vector<uint32_t> rec_mul;
+  std::vector<WarpDesc> units;
+  const uint64_t unit_segs = FR_UNIT_SEGS_PACK;
+  const uint64_t dyn_pct = mix == kSharePack ? FR_DYN_PCT_PACK : 0;
+  const bool claims = mixed && dyn_pct > 0;
   for (ChunkDesc& d : chunks) {
     d.blk_begin = 0;
     d.first_rec = 0;
@@ -299,14 +330,15 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
       const size_t lbase = cl[q].list_off;
       const std::vector<uint64_t>& seg_start = cl[q].seg_start;
       const uint64_t n_seg = seg_start.size() - 1, Wq = wc[q];
+      const uint64_t n_fix = claims ? n_seg - n_seg * dyn_pct / 100 : n_seg;  // segments in the warps' ranges
       SweepClass sc;
       sc.dtype = cls / 2;
       sc.aligned = (cls & 1u) != 0;
       sc.warp_off = warps.size();
       sc.list_off = lbase;
       uint64_t k = 0;  // walks the class list monotonically
-      for (uint64_t w = 0; w < Wq; ++w) {
-        const uint64_t b0 = seg_start[n_seg * w / Wq], b1 = seg_start[n_seg * (w + 1) / Wq];
+      // the descriptor of class blocks [b0, b1), with one record per chunk it overlaps
+      auto range = [&](uint64_t b0, uint64_t b1) {
         WarpDesc wd;
         std::memset(&wd, 0, sizeof wd);
         wd.blk_begin = b0;
@@ -330,12 +362,25 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
             if (bb == end) ++j;
           }
         }
+        return wd;
+      };
+      for (uint64_t w = 0; w < Wq; ++w) {
+        const WarpDesc wd = range(seg_start[n_fix * w / Wq], seg_start[n_fix * (w + 1) / Wq]);
         if (mixed)
           warps[warp_base + slot[q * W + w]] = wd;
         else
           warps.push_back(wd);
       }
-      if (!mixed) bi.classes.push_back(sc);
+      if (mixed) {
+        SweepClass& ms = bi.classes.back();
+        ms.unit_off[cls] = static_cast<uint32_t>(units.size());
+        ms.class_list[cls] = static_cast<uint32_t>(lbase);
+        for (uint64_t u = n_fix; u < n_seg; u += unit_segs)
+          units.push_back(range(seg_start[u], seg_start[std::min(u + unit_segs, n_seg)]));
+        ms.n_units[cls] = static_cast<uint32_t>(units.size() - ms.unit_off[cls]);
+      } else {
+        bi.classes.push_back(sc);
+      }
     }
     D.batches.push_back(bi);
   }
@@ -345,6 +390,12 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
   if (e == cudaSuccess) e = upload(&D.d_lists, lists);
   if (e == cudaSuccess) e = upload(&D.d_rec_nblk, rec_nblk);
   if (e == cudaSuccess) e = upload(&D.d_rec_mul, rec_mul);
+  if (e == cudaSuccess) e = upload(&D.d_units, units);
+  if (e == cudaSuccess && claims) {
+    const size_t qbytes = kQueueWords * sizeof(uint32_t) * std::max<size_t>(D.batches.size(), 1);
+    e = cudaMalloc(&D.d_queue, qbytes);
+    if (e == cudaSuccess) e = cudaMemset(D.d_queue, 0, qbytes);
+  }
   const uint64_t slots = std::max<uint64_t>(D.n_recs, min_recs);
   if (e == cudaSuccess && slots) e = cudaMalloc(&D.d_recs, slots * sizeof(Record));
   return e;
@@ -358,11 +409,18 @@ fr_status run_batches(fr_plan p, const Decomp& D, int mode, uint8_t* packed, FpE
       SweepParams sp;
       sp.chunks = D.d_chunks;
       sp.warps = D.d_warps + sc.warp_off;
-      sp.class_chunks = D.d_lists + sc.list_off;
+      sp.class_chunks = D.d_lists;  // (WarpDesc::list_off is absolute)
       sp.recs = D.d_recs;
       sp.segs = p->d_segs;
       sp.packed = packed;
       sp.n_warps = D.n_warps;
+      sp.units = D.d_units;
+      sp.queue = D.d_queue ? D.d_queue + kQueueWords * b : nullptr;
+      for (uint32_t c = 0; c < kClassCount; ++c) {
+        sp.unit_off[c] = sc.unit_off[c];
+        sp.n_units[c] = sc.n_units[c];
+        sp.list_off[c] = sc.class_list[c];
+      }
       cudaError_t e;
       if (D.mixed)
         e = mode == kModeFingerprint ? launch_sweep_fp_mixed(sp, D.n_ctas, s)

@@ -27,6 +27,17 @@ struct SweepParams {
   double* segs;           // segment sums of squares (all modes but kModeUnpack)
   uint8_t* packed;        // pack: destination; unpack: source; fingerprint: unused
   uint32_t n_warps;       // warps with a descriptor
+  // Mixed launches: per sweep class c, n_units[c] work units at
+  // units + unit_off[c] (block order), claimed at run time by warps that have
+  // finished their own range, and list_off[c], where the class's chunk list
+  // starts.  queue[c] counts the claims on class c, queue[kClassCount] the
+  // warps that have left; all are zero when a launch starts and the last warp
+  // to leave puts them back to zero.  queue = null: no units.
+  const WarpDesc* units;
+  uint32_t* queue;
+  uint32_t unit_off[kClassCount];
+  uint32_t n_units[kClassCount];
+  uint32_t list_off[kClassCount];
 };
 
 struct FinalizeParams {

@@ -52,6 +52,8 @@ constexpr uint32_t kMagic = 0x31435246u;  // bytes 'F','R','C','1'
 constexpr uint32_t kVersion = 1;
 
 enum : uint32_t { kDtBytes = 0, kDtBf16 = 1, kDtF32 = 2 };
+// Sweep classes: element type * 2 + (tensor 16-byte aligned ? 1 : 0).
+constexpr uint32_t kClassCount = 6;
 
 struct ChunkDesc {       // 64 bytes
   uint64_t addr;         // device address of the chunk's first byte in its tensor

@@ -246,6 +246,9 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
     sp.segs = reinterpret_cast<double*>(scratch + kOffSegs);
     sp.packed = nullptr;
     sp.n_warps = static_cast<uint32_t>(W);
+    sp.units = nullptr;  // the warps' ranges cover every block: no claimed units
+    sp.queue = nullptr;
+    for (uint32_t c = 0; c < kClassCount; ++c) sp.unit_off[c] = sp.n_units[c] = sp.list_off[c] = 0;
     e = launch_sweep_fp_mixed(sp, n_sm, s);
     if (e != cudaSuccess) return fail(e);
   }

@@ -622,6 +622,21 @@ __device__ __forceinline__ void sweep_piece_al(const uint8_t* tensor, uint8_t* p
     sweep_piece<MODE, DT, AL, 16>(tensor, packed, n, lane, rec, segs);
 }
 
+// Claims the next unit of class c for this warp: its index within the
+// class's units, or n_units[c] when none is left.
+__device__ __forceinline__ uint32_t claim_unit(const SweepParams& p, uint32_t c, uint32_t lane) {
+  uint32_t u = 0;
+  if (lane == 0) u = atomicAdd(p.queue + c, 1u);
+  return __shfl_sync(0xFFFFFFFFu, u, 0);
+}
+
+// Whether a mode's mixed launches take claimed units: pack and unpack, which
+// are bound by memory latency and whose warps' rates differ from SM to SM by
+// a few percent.  The issue-bound fingerprint keeps its static split: the
+// claim loop around its sweep costs it more registers than the tail it
+// would save.
+__host__ __device__ constexpr bool mode_claims(int m) { return m != kModeFingerprint; }
+
 // One warp's range of its class's block stream: the pieces it overlaps, in
 // order.  ALIGNED: every tensor of the class is 16-byte aligned (128-bit
 // loads and stores); else the tensor side uses 32-bit or byte accesses, chosen
@@ -653,6 +668,24 @@ __device__ __forceinline__ void sweep_warp(const SweepParams& p, const WarpDesc&
   }
 }
 
+// One warp's range, then (pack and unpack launches with units, p.queue set)
+// the units of sweep class `cls` it claims, one at a time, until none is
+// left.  (Plain unpack runs every element type as bytes, so `cls` names the
+// class's queue, not the code.)
+template <int MODE, int DT, bool ALIGNED>
+__device__ __forceinline__ void sweep_warp_claims(const SweepParams& p, const WarpDesc& wd, uint32_t cls,
+                                                  uint32_t lane) {
+  const uint32_t* class_chunks = p.class_chunks + wd.list_off;
+  WarpDesc cur = wd;
+  for (;;) {
+    sweep_warp<MODE, DT, ALIGNED>(p, cur, class_chunks, lane);
+    if (p.queue == nullptr) return;
+    const uint32_t u = claim_unit(p, cls, lane);
+    if (u >= p.n_units[cls]) return;
+    cur = p.units[p.unit_off[cls] + u];
+  }
+}
+
 // One kernel per (mode, element type, alignment class).
 template <int MODE, int DT, bool ALIGNED>
 __global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_kernel(SweepParams p) {
@@ -664,33 +697,85 @@ __global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_kernel(SweepPara
   sweep_warp<MODE, DT, ALIGNED>(p, p.warps[w], p.class_chunks, lane);
 }
 
+// Class c's code for this mode: plain unpack only copies and checksums, so
+// it runs every element type as bytes.
+template <int MODE, uint32_t C>
+__device__ __forceinline__ void sweep_class(const SweepParams& p, const WarpDesc& wd, uint32_t lane) {
+  constexpr int DT = mode_sums(MODE) ? static_cast<int>(C / 2) : static_cast<int>(kDtBytes);
+  sweep_warp_claims<MODE, DT, (C & 1u) != 0>(p, wd, C, lane);
+}
+
+// Help with class c's units left once a warp's own class has none.
+template <int MODE, uint32_t C>
+__device__ __forceinline__ void help_class(const SweepParams& p, uint32_t lane) {
+  if (p.n_units[C] == 0) return;
+  WarpDesc none;
+  none.blk_begin = 0;
+  none.nblk = 0;
+  none.first_chunk = 0;
+  none.rec_base = 0;
+  none.cls = C;
+  none.list_off = p.list_off[C];
+  sweep_class<MODE, C>(p, none, lane);
+}
+
 // Every class of a batch in one launch: each warp sweeps a range of its own
-// class (wd.cls, chunk list at class_chunks + wd.list_off), and the plan
-// spreads each class's warps over all CTAs, so warps that wait on memory and
-// warps that are bound by instruction issue share every SM.
+// class, and the plan spreads each class's warps over all CTAs, so warps that
+// wait on memory and warps that are bound by instruction issue share every
+// SM.  The ranges cover most of each class's blocks; the rest is cut into
+// small units that warps claim one at a time once their own range is done:
+// first their own class's, then, in a fixed order, every other class's, so
+// the launch ends when the work does, not when its slowest warp does.  Which
+// warp sweeps a unit changes nothing in the results: a unit's records and
+// segment sums have fixed slots.  (The class code is inlined once per call
+// site and no loop runs over classes: a loop around the inlined sweeps makes
+// the compiler keep every variant's registers live at once.)
 template <int MODE>
 __global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_mixed_kernel(SweepParams p) {
   fill_tables();
   __syncthreads();
   const uint32_t lane = threadIdx.x & 31u;
   const uint32_t w = blockIdx.x * Cta<MODE>::kWarps + (threadIdx.x >> 5);
-  if (w >= p.n_warps) return;
-  const WarpDesc wd = p.warps[w];
-  const uint32_t* list = p.class_chunks + wd.list_off;
-  if constexpr (!mode_sums(MODE)) {  // (copies and checksums bytes only: no element types)
-    if (wd.cls & 1u)
-      sweep_warp<MODE, kDtBytes, true>(p, wd, list, lane);
-    else
-      sweep_warp<MODE, kDtBytes, false>(p, wd, list, lane);
-    return;
-  }
-  switch (wd.cls) {
-    case kDtF32 * 2 + 1: sweep_warp<MODE, kDtF32, true>(p, wd, list, lane); break;
-    case kDtBf16 * 2 + 1: sweep_warp<MODE, kDtBf16, true>(p, wd, list, lane); break;
-    case kDtBytes * 2 + 1: sweep_warp<MODE, kDtBytes, true>(p, wd, list, lane); break;
-    case kDtF32 * 2: sweep_warp<MODE, kDtF32, false>(p, wd, list, lane); break;
-    case kDtBf16 * 2: sweep_warp<MODE, kDtBf16, false>(p, wd, list, lane); break;
-    default: sweep_warp<MODE, kDtBytes, false>(p, wd, list, lane); break;
+  if constexpr (!mode_claims(MODE)) {
+    // the static split: each warp its own range, one dispatch on its class
+    if (w >= p.n_warps) return;
+    const WarpDesc wd = p.warps[w];
+    const uint32_t* list = p.class_chunks + wd.list_off;
+    switch (wd.cls) {
+      case kDtF32 * 2 + 1: sweep_warp<MODE, kDtF32, true>(p, wd, list, lane); break;
+      case kDtBf16 * 2 + 1: sweep_warp<MODE, kDtBf16, true>(p, wd, list, lane); break;
+      case kDtBytes * 2 + 1: sweep_warp<MODE, kDtBytes, true>(p, wd, list, lane); break;
+      case kDtF32 * 2: sweep_warp<MODE, kDtF32, false>(p, wd, list, lane); break;
+      case kDtBf16 * 2: sweep_warp<MODE, kDtBf16, false>(p, wd, list, lane); break;
+      default: sweep_warp<MODE, kDtBytes, false>(p, wd, list, lane); break;
+    }
+  } else {
+    if (w < p.n_warps) {
+      const WarpDesc wd = p.warps[w];
+      switch (wd.cls) {
+        case kDtF32 * 2 + 1: sweep_class<MODE, kDtF32 * 2 + 1>(p, wd, lane); break;
+        case kDtBf16 * 2 + 1: sweep_class<MODE, kDtBf16 * 2 + 1>(p, wd, lane); break;
+        case kDtBytes * 2 + 1: sweep_class<MODE, kDtBytes * 2 + 1>(p, wd, lane); break;
+        case kDtF32 * 2: sweep_class<MODE, kDtF32 * 2>(p, wd, lane); break;
+        case kDtBf16 * 2: sweep_class<MODE, kDtBf16 * 2>(p, wd, lane); break;
+        default: sweep_class<MODE, kDtBytes * 2>(p, wd, lane); break;
+      }
+    }
+    if (p.queue == nullptr) return;
+    help_class<MODE, kDtF32 * 2 + 1>(p, lane);
+    help_class<MODE, kDtBf16 * 2 + 1>(p, lane);
+    help_class<MODE, kDtBytes * 2 + 1>(p, lane);
+    help_class<MODE, kDtF32 * 2>(p, lane);
+    help_class<MODE, kDtBf16 * 2>(p, lane);
+    help_class<MODE, kDtBytes * 2>(p, lane);
+    // Every warp has made its last claim once it gets here; the last one out
+    // zeroes the queue for the next launch on this plan.
+    if (lane == 0) {
+      __threadfence();
+      if (atomicAdd(p.queue + kClassCount, 1u) == gridDim.x * Cta<MODE>::kWarps - 1) {
+        for (uint32_t c = 0; c <= kClassCount; ++c) atomicExch(p.queue + c, 0u);
+      }
+    }
   }
 }
 
