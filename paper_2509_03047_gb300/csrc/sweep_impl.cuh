@@ -103,12 +103,29 @@ extern __shared__ __align__(16) uint8_t g_smem[];
 //   (k >> 1) * 65536 + i * 256 + (k & 1) * 128 + l * 4,
 // i.e. bank l.  The address of (table k, byte k of x, this lane) is one
 // byte-permute: byte 0 = l*4, byte 1 = byte k of x.
+// Every thread of a kThreads-thread CTA stores its share of 16-byte units;
+// the loop is unrolled so a thread's table loads all issue before the first
+// store waits on one (a rolled loop made the fill a chain of ~16 L2 round
+// trips, about 3 us per launch).
+template <int kThreads>
 __device__ __forceinline__ void fill_tables() {
-  for (int q = threadIdx.x; q < kTableBytes / 16; q += blockDim.x) {
-    const int k = q >> 11, rem = q & 2047, i = rem >> 3, g = rem & 7;
-    const uint32_t v = g_braid.t[k][i];
-    const uint32_t off = (k >> 1) * 65536 + i * 256 + (k & 1) * 128 + g * 16;
-    *reinterpret_cast<uint4*>(g_smem + off) = make_uint4(v, v, v, v);
+  constexpr int kUnits = kTableBytes / 16;
+  constexpr int kIters = (kUnits + kThreads - 1) / kThreads;
+  uint32_t v[kIters];
+#pragma unroll
+  for (int it = 0; it < kIters; ++it) {
+    const int q = static_cast<int>(threadIdx.x) + it * kThreads;
+    const int k = q >> 11, i = (q & 2047) >> 3;
+    v[it] = q < kUnits ? g_braid.t[k][i] : 0u;
+  }
+#pragma unroll
+  for (int it = 0; it < kIters; ++it) {
+    const int q = static_cast<int>(threadIdx.x) + it * kThreads;
+    if (q < kUnits) {
+      const int k = q >> 11, rem = q & 2047, i = rem >> 3, g = rem & 7;
+      const uint32_t off = (k >> 1) * 65536 + i * 256 + (k & 1) * 128 + g * 16;
+      *reinterpret_cast<uint4*>(g_smem + off) = make_uint4(v[it], v[it], v[it], v[it]);
+    }
   }
 }
 
@@ -689,7 +706,7 @@ __device__ __forceinline__ void sweep_warp_claims(const SweepParams& p, const Wa
 // One kernel per (mode, element type, alignment class).
 template <int MODE, int DT, bool ALIGNED>
 __global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_kernel(SweepParams p) {
-  fill_tables();
+  fill_tables<Cta<MODE>::kThreads>();
   __syncthreads();
   const uint32_t lane = threadIdx.x & 31u;
   const uint32_t w = blockIdx.x * Cta<MODE>::kWarps + (threadIdx.x >> 5);
@@ -732,7 +749,7 @@ __device__ __forceinline__ void help_class(const SweepParams& p, uint32_t lane) 
 // the compiler keep every variant's registers live at once.)
 template <int MODE>
 __global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) sweep_mixed_kernel(SweepParams p) {
-  fill_tables();
+  fill_tables<Cta<MODE>::kThreads>();
   __syncthreads();
   const uint32_t lane = threadIdx.x & 31u;
   const uint32_t w = blockIdx.x * Cta<MODE>::kWarps + (threadIdx.x >> 5);
@@ -795,7 +812,7 @@ __device__ __noinline__ void list_piece(const uint8_t* tensor, uint8_t* packed, 
 
 template <int MODE>
 __global__ void __launch_bounds__(Cta<MODE>::kThreads, 1) list_kernel(ListParams p) {
-  fill_tables();
+  fill_tables<Cta<MODE>::kThreads>();
   __syncthreads();
   const uint32_t lane = threadIdx.x & 31u;
   const uint64_t w = static_cast<uint64_t>(blockIdx.x) * Cta<MODE>::kWarps + (threadIdx.x >> 5);
