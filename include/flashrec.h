@@ -36,7 +36,12 @@
  *     The caller owns every tensor, buffer and output; the library owns only
  *     the plan and what the plan allocates when it is created.  No call after
  *     fr_plan_create allocates memory.
- *   - Thread safety: a plan may be used by one stream at a time.
+ *   - Thread safety: a plan may be used by one stream at a time.  Calls on
+ *     one plan whose kernels overlap on the GPU (the same plan on two streams
+ *     with no ordering between them) race on the plan's scratch -- per-piece
+ *     records, segment sums and the counters through which pack and unpack
+ *     warps share their last work units -- and give wrong results.  (The
+ *     batched calls of a batched plan have their own counters per batch.)
  */
 #ifndef FLASHREC_H
 #define FLASHREC_H
