@@ -45,19 +45,31 @@ KERNEL_FILES = ["sweep_fp.cu", "sweep_pack.cu", "sweep_unpack.cu", "sweep_unpack
                 "layout.h", "kernels.h", "sweep_impl.cuh"]
 
 
+def _code_only(text: str) -> str:
+    """`text` without its C/C++ comments, trailing blanks and blank lines:
+    what the compiler sees, so an edit to a comment leaves the digest alone.
+    (String literals in these sources contain no comment markers.)"""
+    import re
+
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", "", text)
+    return "\n".join(line.rstrip() for line in text.splitlines() if line.strip())
+
+
 def source_digest(kernels_only: bool = False) -> str:
-    """Hash of the sources and compile flags (identifies what a profile
-    measured); with `kernels_only`, of the device-kernel files alone."""
+    """Hash of the sources' code (comments left out) and the compile flags:
+    identifies what a profile measured.  With `kernels_only`, of the
+    device-kernel files alone."""
     import hashlib
 
     h = hashlib.sha256(" ".join(a for a in ARCH + NVCC_FLAGS if not os.path.isabs(a)).encode())
     names = KERNEL_FILES if kernels_only else SOURCES + HEADERS
     for name in sorted(names):
-        with open(os.path.join(CSRC, name), "rb") as f:
-            h.update(name.encode() + b"\0" + f.read())
+        with open(os.path.join(CSRC, name), encoding="utf-8") as f:
+            h.update(name.encode() + b"\0" + _code_only(f.read()).encode())
     if not kernels_only:
-        with open(os.path.join(ROOT, "include", "flashrec.h"), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, "include", "flashrec.h"), encoding="utf-8") as f:
+            h.update(_code_only(f.read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -19,19 +19,20 @@
 //    square is added to a packed f32x2 running sum by one FMA, and the
 //    addition's error -- including the square's own rounding for fp32 -- is
 //    recovered to second order by a TwoSum whose low term is a second FMA
-//    (two_sum_sq), then flushed into fp64.  A
-//    stage whose running sum is not finite (NaN/Inf input, or overflow) or is
-//    tiny with non-zero input is discarded and redone element by element in
-//    fp64 from a reload of its 16-byte units, so the fast path never needs a
-//    per-element test.
+//    (two_sum_sq), then flushed into fp64.  A 16 KiB segment whose running
+//    sum is not finite (NaN/Inf input, or overflow) or is tiny with non-zero
+//    input is redone element by element in fp64 from a reload of its 16-byte
+//    units, so the fast path never needs a per-element test.
 //
 // No tensor cores: nothing here is a contraction.  One CTA per SM, with a warp
 // count per mode (the 128 KiB of lane-replicated tables fill most of shared
-// memory).  The
-// plan sorts chunks into classes by element type and by whether the tensor
-// is 16-byte aligned; each class gets its own block stream, cut into equal
-// per-warp ranges, and its own kernel specialization, so every kernel holds a
-// single loop variant and its registers.  sweep_{fp,pack,unpack}.cu each
+// memory).  The plan sorts chunks into classes by element type and by whether
+// the tensor is 16-byte aligned; each class has its own block stream, cut
+// into per-warp ranges, and its own code specialization, so each warp runs a
+// single loop variant.  A call launches once for all its classes
+// (sweep_mixed_kernel: each warp dispatches on its range's class once);
+// pack and unpack warps then claim the last few percent of the work as small
+// units (see sweep_warp_claims).  sweep_{fp,pack,unpack,unpack_fp}.cu each
 // instantiate one mode.
 #pragma once
 
