@@ -324,7 +324,11 @@ fr_status fr_shard_pieces(uint64_t n_elems, uint32_t elem_bytes, uint32_t n_dst,
  *     results.  Host-side calls are serialized by a lock.
  *   - The table upload is a copy from pageable host memory, so the call
  *     returns only after the work already queued on `stream` has finished.
- * Errors: FR_ERR_INVALID_ARG (also for sizes beyond the limit), FR_ERR_CUDA. */
+ *   - It cannot be captured into a CUDA graph (a replay would upload whatever
+ *     tables the latest call left in the host buffer): on a stream under
+ *     capture it returns FR_ERR_INVALID_ARG and enqueues nothing.
+ * Errors: FR_ERR_INVALID_ARG (also for sizes beyond the limit, or a stream
+ * under capture), FR_ERR_CUDA. */
 #define FR_STATIC_MAX_CHUNKS 16384
 #define FR_STATIC_MAX_SEGMENTS 131072
 fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_tensors, uint64_t chunk_bytes,

@@ -45,11 +45,9 @@ constexpr int kFinWarps = 8;
 constexpr int kFinThreads = kFinWarps * 32;
 constexpr unsigned kFull = 0xFFFFFFFFu;
 
-__device__ const ByteTable g_byte = make_byte_table();
 __device__ const PowTables g_pow = make_pow_tables();
 // Byte tables for multiplying by the constants x^(32 * 2^k), k = 0..6
-// (x^32 ... x^2048): the shuffle trees that join 4-byte header words and
-// 16-byte tail pieces lane by lane.
+// (x^32 ... x^2048); the tail's CRC uses x^1024 and x^2048.
 struct ConstMulTables {
   ByteTables4 m[7];
 };
@@ -67,30 +65,54 @@ __device__ __forceinline__ uint32_t mul_x32k(int k, uint32_t a) {
          (__ldg(&T.t[2][(a >> 16) & 255u]) ^ __ldg(&T.t[3][a >> 24]));
 }
 
-// Joins the raw CRCs v of lanes 0..2^levels-1, lane l holding piece l of
-// 4 * 2^first bytes each, in lane order: lane 0 ends with raw(piece 0 || ... ).
-__device__ __forceinline__ uint32_t join_lanes(uint32_t v, int first, int levels) {
-  for (int j = 0; j < levels; ++j) {
-    const uint32_t o = __shfl_down_sync(kFull, v, 1u << j);
-    v = mul_x32k(first + j, v) ^ o;
+// Per-lane multipliers.  In a 128-word window whose word i goes to lane
+// i % 32, a word of lane l has (31 - l) + 32j words after it, j fixed by its
+// slot, so lane l's partial CRC takes the shift M_l = x^(32 (32 - l)) (the
+// word's own x^32 included) before the lanes are XORed together.  The
+// product (n << 4k) * M_l, for nibble position k and nibble value n, sits at
+// word (16k + n) * 32 + l: the 32 lanes' lookups of one nibble position fall
+// in 32 different shared-memory banks.  16 KiB.
+constexpr int kLaneMulWords = 8 * 16 * 32;
+struct alignas(16) LaneMulTable {
+  uint32_t t[kLaneMulWords];
+};
+__host__ __device__ constexpr LaneMulTable make_lane_mul_table() {
+  LaneMulTable out{};
+  for (int l = 0; l < 32; ++l) {
+    const uint32_t m = gf_xpow(32ull * static_cast<uint64_t>(32 - l));
+    for (int k = 0; k < 8; ++k) {
+      uint32_t bit[4] = {};
+      for (int j = 0; j < 4; ++j) bit[j] = gf_mulmod(1u << (4 * k + j), m);
+      for (int n = 0; n < 16; ++n) {
+        uint32_t v = 0;
+        for (int j = 0; j < 4; ++j)
+          if (n & (1 << j)) v ^= bit[j];
+        out.t[(16 * k + n) * 32 + l] = v;
+      }
+    }
   }
-  return v;
+  return out;
+}
+__device__ const LaneMulTable g_lane_mul = make_lane_mul_table();
+
+// a * M_l mod P for the calling lane l; `LM` is the shared copy of the table
+// offset by the lane.
+__device__ __forceinline__ uint32_t lane_mul(const uint32_t* LM, uint32_t a) {
+  uint32_t r[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) r[k] = LM[(16 * k + ((a >> (4 * k)) & 15u)) * 32];
+  return (r[0] ^ r[1] ^ r[2]) ^ (r[3] ^ r[4] ^ r[5]) ^ (r[6] ^ r[7]);
 }
 
-// CRC-32C of the 60 header bytes given as 15 words, computed by lanes 1..15
-// (lane l CRCs word l-1; lane 0 is a leading zero word, which leaves a raw
-// CRC run from zero unchanged) and joined in a 4-level tree; all lanes return
-// it.  `T` is the byte table.
-__device__ __forceinline__ uint32_t header_crc(const uint32_t* T, const uint32_t h[15], uint32_t lane) {
+// CRC-32C of the 60 header bytes given as 15 words: word k (followed by
+// 14 - k more) sits in lane 17 + k, whose multiplier M_(17+k) = x^(32 (15 - k))
+// is exactly its shift; every lane returns it.
+__device__ __forceinline__ uint32_t header_crc(const uint32_t* LM, const uint32_t h[15], uint32_t lane) {
   uint32_t w = 0;
 #pragma unroll
-  for (int k = 0; k < 15; ++k) w = (lane == static_cast<uint32_t>(k + 1)) ? h[k] : w;
-  uint32_t r = 0;
-#pragma unroll
-  for (int j = 0; j < 4; ++j) r = T[(r ^ (w >> (8 * j))) & 0xFFu] ^ (r >> 8);
-  const uint32_t raw = join_lanes(lane < 16 ? r : 0u, 0, 4);
+  for (int k = 0; k < 15; ++k) w = (lane == static_cast<uint32_t>(17 + k)) ? h[k] : w;
   constexpr uint32_t kHeaderXor = gf_mulmod(0xFFFFFFFFu, gf_xpow(8 * 60)) ^ 0xFFFFFFFFu;
-  return __shfl_sync(kFull, raw, 0) ^ kHeaderXor;
+  return __reduce_xor_sync(kFull, lane_mul(LM, w)) ^ kHeaderXor;
 }
 
 // a * b mod P, both variable.
@@ -131,8 +153,9 @@ __device__ __forceinline__ void two_sum_pair(float& hi, float& lo, float bh, flo
 // One tail element of type `dtype` with bit pattern `bits`: counted if
 // non-finite, else its square added exactly -- as an fp32 product and its FMA
 // residual into the float pair (hi, lo) when |x| lies in [2^-40, 2^56] (the
-// residual is not subnormal, and 32 lanes of 8 squares stay below 2^120), else
-// in fp64 into dx (rare).  The common case stays off GB300's narrow fp64 pipe.
+// residual is not subnormal, and a lane's 8 squares add at most 2^115), else
+// in fp64 into dx (rare).  The common case stays off GB300's narrow fp64
+// pipe.
 __device__ __forceinline__ void tail_elem(uint32_t dtype, uint32_t bits, uint32_t& nf, float& hi, float& lo,
                                           double& dx) {
   uint32_t f;
@@ -154,23 +177,35 @@ __device__ __forceinline__ void tail_elem(uint32_t dtype, uint32_t bits, uint32_
   }
 }
 
-// Adds one segment slot (see seg_value) to the float pair (hi, lo) or, in the
-// tagged fp64 form, to dx.
+// Adds one segment slot (see seg_value) to the float pair (hi, lo), or to dx
+// in fp64 if it is in the tagged fp64 form or its sum is 2^90 or more (rare):
+// a lane's float pair then stays below 2^119 for any chunk of fewer than 2^47
+// bytes, tail squares included, and the 32-lane tree cannot overflow.
 __device__ __forceinline__ void add_slot(uint64_t bits, float& hi, float& lo, double& dx) {
+  const float bh = __uint_as_float(static_cast<uint32_t>(bits >> 32));
+  const float bl = __uint_as_float(static_cast<uint32_t>(bits));
   if (bits >> 63)
     dx += -__longlong_as_double(static_cast<long long>(bits));
+  else if (bh < 0x1p90f)
+    two_sum_pair(hi, lo, bh, bl);
   else
-    two_sum_pair(hi, lo, __uint_as_float(static_cast<uint32_t>(bits >> 32)), __uint_as_float(static_cast<uint32_t>(bits)));
+    dx += static_cast<double>(bh) + static_cast<double>(bl);
 }
 
 __device__ __forceinline__ void prefetch_l1(const void* q) { asm volatile("prefetch.global.L1 [%0];" ::"l"(q)); }
 
 template <int MODE>
 __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(FinalizeParams p) {
-  __shared__ uint32_t T[256];
-  for (int i = threadIdx.x; i < 256; i += kFinThreads) T[i] = g_byte.t[i];
+  __shared__ LaneMulTable lm_s;
+  {
+    const uint4* src = reinterpret_cast<const uint4*>(g_lane_mul.t);
+    uint4* dst = reinterpret_cast<uint4*>(lm_s.t);
+#pragma unroll
+    for (int i = 0; i < kLaneMulWords / 4 / kFinThreads; ++i) dst[threadIdx.x + i * kFinThreads] = src[threadIdx.x + i * kFinThreads];
+  }
   __syncthreads();
   const uint32_t lane = threadIdx.x & 31u;
+  const uint32_t* LM = lm_s.t + lane;
   const uint64_t stride = static_cast<uint64_t>(gridDim.x) * kFinWarps;
   for (uint64_t pos = p.c_begin + static_cast<uint64_t>(blockIdx.x) * kFinWarps + (threadIdx.x >> 5);
        pos < p.c_end; pos += stride) {
@@ -207,20 +242,36 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
       tsrc = reinterpret_cast<const uint8_t*>(cd.addr) + body;
       if (MODE == kModePack) tdst = p.packed + cd.payload_off + body;
     }
-    // lane l takes the 16 tail bytes that end 16 * (31 - l) bytes before the
-    // tail's end, as four little-endian words; bytes before the tail read as
-    // zeros (leading zero bytes leave a raw CRC run from zero unchanged and
-    // add nothing to the sums), so the lane's shift is a constant
-    const int32_t e0 = static_cast<int32_t>(tail) - 16 * (32 - static_cast<int32_t>(lane));
+    // The tail is read as the end of a 512-byte window whose first z = 512 -
+    // tail bytes are zeros (leading zero bytes leave a raw CRC run from zero
+    // unchanged and add nothing to the sums).  Window word i (bytes 4i..4i+3,
+    // little-endian) is word i / 32 of lane i % 32, so one load instruction
+    // covers 32 consecutive words.  Words are loaded whole when the tail's
+    // end is 4-byte aligned on both sides (a word holding the tail's first
+    // byte then goes byte by byte), else every word byte by byte.
+    const int32_t z = kBlockBytes - static_cast<int32_t>(tail);
+    const bool wordy = ((reinterpret_cast<uintptr_t>(tsrc) + tail) & 3u) == 0 &&
+                       (tdst == nullptr || ((reinterpret_cast<uintptr_t>(tdst) + tail) & 3u) == 0);
     uint32_t w[4] = {0u, 0u, 0u, 0u};
     if (tail != 0) {
 #pragma unroll
-      for (int j = 0; j < 16; ++j)
-        if (e0 + j >= 0) w[j >> 2] |= static_cast<uint32_t>(__ldg(tsrc + (e0 + j))) << (8 * (j & 3));
+      for (int q = 0; q < 4; ++q) {
+        const int32_t t = 4 * (32 * q + static_cast<int32_t>(lane)) - z;  // the word's offset in the tail
+        if (wordy && t >= 0) {
+          w[q] = __ldg(reinterpret_cast<const uint32_t*>(tsrc + t));
+        } else if (t > -4) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (t + j >= 0) w[q] |= static_cast<uint32_t>(__ldg(tsrc + (t + j))) << (8 * j);
+        }
+      }
     }
     const uint32_t crc_xor = p.crc_xor ? p.crc_xor[c] : 0u;
+    // padding after the payload: [pad_begin, pad_end), pad_end 256-aligned,
+    // covered as whole words from pad_begin rounded down to 4 bytes
     const uint64_t pad_begin = cd.payload_off + cd.len;
     const uint64_t pad_end = cd.payload_off + align_up(cd.len, kPayloadAlign);
+    const uint64_t pad_w0 = pad_begin & ~static_cast<uint64_t>(3);
     uint32_t h[16];
     uint32_t pad = 0;  // OR of the padding bytes after the payload (< 256 of them)
     if (mode_unpacks(MODE)) {
@@ -233,10 +284,29 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
         h[4 * q + 2] = v.z;
         h[4 * q + 3] = v.w;
       }
+      const uint32_t* pw = reinterpret_cast<const uint32_t*>(p.packed + pad_w0);
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const uint64_t j = pad_begin + lane + 32u * q;
-        if (j < pad_end) pad |= p.packed[j];
+      for (int q = 0; q < 3; ++q) {
+        const uint32_t k = lane + 32u * q;
+        if (pad_w0 + 4u * k < pad_end) {
+          uint32_t v = pw[k];
+          if (k == 0) v &= 0xFFFFFFFFu << (8 * (pad_begin & 3u));  // payload bytes before pad_begin
+          pad |= v;
+        }
+      }
+    }
+    // pack and unpack copy the tail (before the body's CRC is folded into it)
+    if (tdst != nullptr && tail != 0) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int32_t t = 4 * (32 * q + static_cast<int32_t>(lane)) - z;
+        if (wordy && t >= 0) {
+          *reinterpret_cast<uint32_t*>(tdst + t) = w[q];
+        } else if (t > -4) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (t + j >= 0) tdst[t + j] = static_cast<uint8_t>(w[q] >> (8 * j));
+        }
       }
     }
 
@@ -244,24 +314,19 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
     // -- a multiplier the plan precomputed (1 for the last record, whose
     // multiply is skipped), or (list mode, no-allocation entry) found here,
     // last batch of 32 first so the byte count after each is known
-    uint32_t raw = 0;
-    double sq_rec = 0.0;
-    uint32_t nf_rec = 0;
+    uint32_t raw = 0;      // this lane's share of the body's raw CRC
+    uint32_t nf_lane = 0;  // this lane's share of the non-finite count
     uint64_t carry = 0;
     if (rec_mul) {
-      uint32_t n = 0;
       if (lane < n_recs) {
         raw = mul0 == kOne ? rec0.crc : gmul(rec0.crc, mul0);
-        n = rec0.nonfinite;
+        nf_lane = rec0.nonfinite;
       }
       for (int64_t i = lane + 32; i < n_recs; i += 32) {
         const Record rec = p.recs[first_rec + i];
         raw ^= gmul(rec.crc, p.rec_mul[first_rec + i]);
-        n += rec.nonfinite;
+        nf_lane += rec.nonfinite;
       }
-#pragma unroll
-      for (int m = 16; m >= 1; m >>= 1) n += __shfl_down_sync(kFull, n, m);
-      nf_rec = __shfl_sync(kFull, n, 0);
     }
     for (int64_t hi = rec_mul ? 0 : n_recs; hi > 0;) {
       const int64_t lo = hi > 32 ? hi - 32 : 0;
@@ -281,101 +346,88 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
       }
       if (have) raw ^= shift_bytes(rec.crc, carry + suf - len);
       carry += __shfl_sync(kFull, suf, 0);
-      uint32_t n = rec.nonfinite;
-#pragma unroll
-      for (int m = 16; m >= 1; m >>= 1) n += __shfl_down_sync(kFull, n, m);
-      nf_rec += __shfl_sync(kFull, n, 0);
+      nf_lane += rec.nonfinite;
       hi = lo;
     }
     // the body's raw CRC, in every lane
-#pragma unroll
-    for (int m = 16; m >= 1; m >>= 1) raw ^= __shfl_xor_sync(kFull, raw, m);
-    // the body's segment sums, in an order fixed by segment index alone
+    raw = __reduce_xor_sync(kFull, raw);
+
+    // ---- 2. sums of squares: each lane adds its segment slots (in an order
+    // fixed by segment index, so the result does not depend on the plan),
+    // then its tail elements, as a float pair (pair-form slots and tail
+    // squares by TwoSum; tagged fp64 slots and out-of-range squares, both
+    // rare, in fp64), and one fixed tree adds the lanes: the common case
+    // stays off the narrow fp64 pipe
+    double sq = 0.0;
     if (values) {
-      // pair-form slots are added as float pairs (TwoSum), tagged fp64 slots
-      // (rare) in fp64, so the common case stays off the narrow fp64 pipe
       float hi = 0.0f, lo = 0.0f;
       double dx = 0.0;
       if (lane < n_seg) add_slot(slot0, hi, lo, dx);
       for (uint64_t k = lane + 32; k < n_seg; k += 32)
         add_slot(reinterpret_cast<const uint64_t*>(p.segs + cd.seg_base)[k], hi, lo, dx);
+      if (tail != 0) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          if (cd.dtype == kDtF32) {
+            tail_elem(kDtF32, w[q], nf_lane, hi, lo, dx);
+          } else {
+            tail_elem(kDtBf16, w[q] & 0xFFFFu, nf_lane, hi, lo, dx);
+            tail_elem(kDtBf16, w[q] >> 16, nf_lane, hi, lo, dx);
+          }
+        }
+      }
+      // lanes at or past `active` hold zeros: tree levels that would only add
+      // them are skipped (adding (0, 0) changes no bit of the pair)
+      const uint64_t active = tail != 0 ? 32u : n_seg;
 #pragma unroll
       for (int m = 16; m >= 1; m >>= 1) {
-        const float oh = __shfl_down_sync(kFull, hi, m), ol = __shfl_down_sync(kFull, lo, m);
-        two_sum_pair(hi, lo, oh, ol);
+        if (static_cast<uint64_t>(m) < active) {
+          const float oh = __shfl_down_sync(kFull, hi, m), ol = __shfl_down_sync(kFull, lo, m);
+          two_sum_pair(hi, lo, oh, ol);
+        }
       }
       if (__any_sync(kFull, dx != 0.0)) {
 #pragma unroll
         for (int m = 16; m >= 1; m >>= 1) dx += __shfl_down_sync(kFull, dx, m);
       }
-      sq_rec = (static_cast<double>(hi) + static_cast<double>(lo)) + dx;
+      sq = (static_cast<double>(hi) + static_cast<double>(lo)) + dx;
     }
 
-    // ---- 2. tail: copied, its elements summed, CRC'd a word at a time
-    // continuing from the body's raw CRC: a run started from state r equals
-    // one started from zero with r XORed into its first four bytes, so when
-    // the tail's first word is a whole word of one lane's piece (tail length
-    // a multiple of 4: always for fp32) that lane folds the body in there and
-    // the joined tail pieces give raw(body || tail) with no shift of the body;
-    // other tails (byte tensors, bf16) shift the body by x^(8 tail)
-    float th = 0.0f, tl = 0.0f;  // the tail's sum of squares, as a float pair
-    double tdx = 0.0;            // and its rare fp64 part
-    uint32_t nf_tail = 0;
+    // ---- 3. the tail's CRC, continuing the body's: a run started from state
+    // r equals one started from zero with r XORed into its first four bytes,
+    // so when the tail's first byte starts a window word (tail length a
+    // multiple of 4: always for fp32) the body's raw CRC is XORed into that
+    // word and the window's raw CRC is raw(body || tail) with no shift of the
+    // body; other tails (byte tensors, some bf16) shift the body by
+    // x^(8 tail).  Lane l's words w_q (window words 32q + l) combine as
+    // sum_q w_q x^(1024 (3 - q)) (two multiplies by x^1024 and one by
+    // x^2048), then take the lane's shift M_l, and the lanes are XORed.
     if (tail != 0) {
-      uint32_t tail_raw = 0;
-      if (e0 + 16 > 0) {
-        if (tdst) {
-#pragma unroll
-          for (int j = 0; j < 16; ++j)
-            if (e0 + j >= 0) tdst[e0 + j] = static_cast<uint8_t>(w[j >> 2] >> (8 * (j & 3)));
-        }
-        if (values) {
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            if (cd.dtype == kDtF32) {
-              tail_elem(kDtF32, w[q], nf_tail, th, tl, tdx);
-            } else {
-              tail_elem(kDtBf16, w[q] & 0xFFFFu, nf_tail, th, tl, tdx);
-              tail_elem(kDtBf16, w[q] >> 16, nf_tail, th, tl, tdx);
-            }
-          }
-        }
-        if (e0 <= 0) {  // the tail's first byte is in this lane's piece
+      const bool fold = (tail & 3u) == 0;
+      if (fold) {
+        const uint32_t i0 = static_cast<uint32_t>(z) >> 2;  // the window word holding the tail's first byte
+        if (lane == (i0 & 31u)) {
 #pragma unroll
           for (int q = 0; q < 4; ++q)
-            if (4 * q == -e0) w[q] ^= raw;  // only when it starts a word
+            if (static_cast<uint32_t>(q) == (i0 >> 5)) w[q] ^= raw;
         }
-#pragma unroll
-        for (int q = 0; q < 4; ++q) tail_raw = mul_x32k(0, tail_raw ^ w[q]);
       }
-      // lane l's piece ends 16 * (31 - l) bytes before the tail's end: join
-      // the 32 pieces in lane order into lane 0
-      const uint32_t joined = __shfl_sync(kFull, join_lanes(tail_raw, 2, 5), 0);
-      raw = (tail & 3u) == 0 ? joined : (shift_bytes(raw, tail) ^ joined);
-#pragma unroll
-      for (int m = 16; m >= 1; m >>= 1) {
-        nf_tail += __shfl_down_sync(kFull, nf_tail, m);
-        const float oh = __shfl_down_sync(kFull, th, m), ol = __shfl_down_sync(kFull, tl, m);
-        two_sum_pair(th, tl, oh, ol);
-      }
-      if (__any_sync(kFull, tdx != 0.0)) {
-#pragma unroll
-        for (int m = 16; m >= 1; m >>= 1) tdx += __shfl_down_sync(kFull, tdx, m);
-      }
+      const uint32_t H = mul_x32k(6, mul_x32k(5, w[0]) ^ w[1]) ^ (mul_x32k(5, w[2]) ^ w[3]);
+      const uint32_t joined = __reduce_xor_sync(kFull, lane_mul(LM, H));
+      raw = (fold || raw == 0) ? joined : (shift_bytes(raw, tail) ^ joined);
     }
-    const double sq_tail = (static_cast<double>(th) + static_cast<double>(tl)) + tdx;
 
-    // ---- 3. preset and final XOR
+    // ---- 4. preset and final XOR
     const uint32_t crc = raw ^ (p.crc_xor ? crc_xor : (shift_bytes(0xFFFFFFFFu, cd.len) ^ 0xFFFFFFFFu));
-    // lane 0 holds the fixed-order sums and counts: every lane gets them
-    const double sumsq = __shfl_sync(kFull, sq_rec + sq_tail, 0);
-    const uint32_t nonfinite = __shfl_sync(kFull, nf_rec + nf_tail, 0);
+    // lane 0 holds the fixed-order sums; every lane gets them and the count
+    const double sumsq = __shfl_sync(kFull, sq, 0);
+    const uint32_t nonfinite = __reduce_add_sync(kFull, nf_lane);
 
     const uint64_t table_end = p.n_chunks * kHeaderBytes;
     const uint64_t gap_end = align_up(table_end, kPayloadAlign);
     const bool last = (c + 1 == p.n_chunks);
 
-    // ---- 4. outputs
+    // ---- 5. outputs
     if (MODE != kModeUnpack && p.out_fp != nullptr) {  // the fingerprint table (optional for pack, unpack-fp)
       if (lane == 0) {
         FpEntry e;
@@ -387,37 +439,45 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
     }
     if (MODE == kModePack) {
       {
-        uint32_t h[15];
+        uint32_t hd[15];
         const uint64_t sbits = static_cast<uint64_t>(__double_as_longlong(sumsq));
-        h[0] = kMagic;
-        h[1] = kVersion | (cd.dtype << 16);
-        h[2] = static_cast<uint32_t>(c);
-        h[3] = static_cast<uint32_t>(c >> 32);
-        h[4] = cd.tensor_idx;
-        h[5] = crc;
-        h[6] = static_cast<uint32_t>(cd.tensor_off);
-        h[7] = static_cast<uint32_t>(cd.tensor_off >> 32);
-        h[8] = static_cast<uint32_t>(cd.len);
-        h[9] = static_cast<uint32_t>(cd.len >> 32);
-        h[10] = static_cast<uint32_t>(cd.payload_off);
-        h[11] = static_cast<uint32_t>(cd.payload_off >> 32);
-        h[12] = static_cast<uint32_t>(sbits);
-        h[13] = static_cast<uint32_t>(sbits >> 32);
-        h[14] = nonfinite;
-        const uint32_t hcrc = header_crc(T, h, lane);
+        hd[0] = kMagic;
+        hd[1] = kVersion | (cd.dtype << 16);
+        hd[2] = static_cast<uint32_t>(c);
+        hd[3] = static_cast<uint32_t>(c >> 32);
+        hd[4] = cd.tensor_idx;
+        hd[5] = crc;
+        hd[6] = static_cast<uint32_t>(cd.tensor_off);
+        hd[7] = static_cast<uint32_t>(cd.tensor_off >> 32);
+        hd[8] = static_cast<uint32_t>(cd.len);
+        hd[9] = static_cast<uint32_t>(cd.len >> 32);
+        hd[10] = static_cast<uint32_t>(cd.payload_off);
+        hd[11] = static_cast<uint32_t>(cd.payload_off >> 32);
+        hd[12] = static_cast<uint32_t>(sbits);
+        hd[13] = static_cast<uint32_t>(sbits >> 32);
+        hd[14] = nonfinite;
+        const uint32_t hcrc = header_crc(LM, hd, lane);
         if (lane == 0) {
           uint4* dst = reinterpret_cast<uint4*>(p.packed + c * kHeaderBytes);
-          for (int q = 0; q < 3; ++q) dst[q] = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
-          dst[3] = make_uint4(h[12], h[13], h[14], hcrc);
+          for (int q = 0; q < 3; ++q) dst[q] = make_uint4(hd[4 * q], hd[4 * q + 1], hd[4 * q + 2], hd[4 * q + 3]);
+          dst[3] = make_uint4(hd[12], hd[13], hd[14], hcrc);
         }
       }
-      for (uint64_t j = pad_begin + lane; j < pad_end; j += 32) p.packed[j] = 0;
+      // zero padding: the bytes up to the first word boundary one by one,
+      // then whole words
+      const uint64_t pad_w1 = (pad_begin + 3) & ~static_cast<uint64_t>(3);
+      if (pad_begin + lane < pad_w1 && pad_begin + lane < pad_end) p.packed[pad_begin + lane] = 0;
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const uint64_t j = pad_w1 + 4u * (lane + 32u * q);
+        if (j < pad_end) *reinterpret_cast<uint32_t*>(p.packed + j) = 0u;
+      }
       if (last)
         for (uint64_t j = table_end + lane * 16u; j < gap_end; j += 512)
           *reinterpret_cast<uint4*>(p.packed + j) = make_uint4(0, 0, 0, 0);
     } else if (mode_unpacks(MODE)) {  // unpack + verify
       // every lane read the (same) header; check it against the plan
-      const uint32_t hcrc = header_crc(T, h, lane);
+      const uint32_t hcrc = header_crc(LM, h, lane);
       bool bad = (h[15] != hcrc) || h[0] != kMagic || (h[1] & 0xFFFFu) != kVersion || (h[1] >> 16) != cd.dtype ||
                  h[2] != static_cast<uint32_t>(c) || h[3] != static_cast<uint32_t>(c >> 32) ||
                  h[4] != cd.tensor_idx || h[6] != static_cast<uint32_t>(cd.tensor_off) ||
@@ -632,8 +692,16 @@ cudaError_t launch_compact(const Pred& pred, uint64_t n, uint32_t* out, uint64_t
 
 cudaError_t launch_finalize(int mode, const FinalizeParams& p, cudaStream_t s) {
   if (p.c_end <= p.c_begin) return cudaSuccess;
-  uint64_t want = (p.c_end - p.c_begin + kFinWarps - 1) / kFinWarps;
-  const int grid = static_cast<int>(want < 4096 ? want : 4096);
+  // every CTA copies the 16 KiB multiplier table into shared memory, so the
+  // grid is at most one full wave (FR_FIN_MINB CTAs per SM), its warps
+  // looping over the chunks
+  int dev = 0, n_sm = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t cap = static_cast<uint64_t>(n_sm > 0 ? n_sm : 1) * FR_FIN_MINB;
+  const uint64_t want = (p.c_end - p.c_begin + kFinWarps - 1) / kFinWarps;
+  const int grid = static_cast<int>(want < cap ? want : cap);
   if (mode == kModeFingerprint)
     finalize_kernel<kModeFingerprint><<<grid, kFinThreads, 0, s>>>(p);
   else if (mode == kModePack)

@@ -124,8 +124,16 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
   if (n_chunks == 0) return FR_OK;
   if (out_dev == nullptr) return fail("out_dev is null");
 
+  // The table upload reads g_host, which every call rewrites: captured into
+  // a graph, a replay would read whatever plan the last call left there.
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaStreamCaptureStatus capturing = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(s, &capturing);
+  if (e != cudaSuccess) return fail(e);
+  if (capturing != cudaStreamCaptureStatusNone) return fail("the stream is being captured; this call cannot be");
+
   int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return fail(e);
   int n_sm = 0;
   e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
@@ -225,7 +233,6 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
   const uint64_t n_warps = n_cls > 0 ? W : 0;
 
   // ---- tables into the scratch, ordered on the caller's stream
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   e = cudaMemcpyAsync(scratch + kOffChunks, h.chunks, n_chunks * sizeof(ChunkDesc), cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess && n_lists)
     e = cudaMemcpyAsync(scratch + kOffLists, h.lists, n_lists * sizeof(uint32_t), cudaMemcpyHostToDevice, s);

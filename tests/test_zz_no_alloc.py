@@ -59,3 +59,20 @@ def test_static_entry_point_rejects_inputs_beyond_its_limit():
     got = _static_table([ok], 4)
     want = fr.Plan([ok], 4).fingerprint()
     assert torch.equal(got, want)
+
+
+def test_static_entry_point_refuses_a_stream_under_capture():
+    # a graph replay would upload whatever tables the latest call left in the
+    # library's host buffer, so the call refuses capture and enqueues nothing
+    t = torch.randn(8192, device="cuda")
+    out = torch.empty(16 * 2, dtype=torch.uint8, device="cuda")
+    want = fr.Plan([t], 16384).fingerprint()
+    s = torch.cuda.Stream()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        with pytest.raises(fr.FlashrecError) as e:
+            fr.fr_fingerprint_static([t], 16384, out, stream=s)
+    assert e.value.status == fr.FR_ERR_INVALID_ARG
+    assert "captured" in fr.fr_last_error()
+    # the same call outside the capture works
+    assert torch.equal(_static_table([t], 16384), want)
