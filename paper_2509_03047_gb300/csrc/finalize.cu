@@ -150,46 +150,52 @@ __device__ __forceinline__ void two_sum_pair(float& hi, float& lo, float bh, flo
   hi = t;
 }
 
-// One tail element of type `dtype` with bit pattern `bits`: counted if
-// non-finite, else its square added exactly -- as an fp32 product and its FMA
-// residual into the float pair (hi, lo) when |x| lies in [2^-40, 2^56] (the
-// residual is not subnormal, and a lane's 8 squares add at most 2^115), else
-// in fp64 into dx (rare).  The common case stays off GB300's narrow fp64
-// pipe.
-__device__ __forceinline__ void tail_elem(uint32_t dtype, uint32_t bits, uint32_t& nf, float& hi, float& lo,
-                                          double& dx) {
-  uint32_t f;
-  if (dtype == kDtF32) {
-    if ((bits & 0x7F800000u) == 0x7F800000u) { ++nf; return; }
-    f = bits;
-  } else {
-    if ((bits & 0x7F80u) == 0x7F80u) { ++nf; return; }
-    f = bits << 16;
-  }
-  const float x = __uint_as_float(f);
-  const float ax = fabsf(x);
-  if (ax >= 0x1p-40f && ax <= 0x1p56f) {
-    const float p2 = x * x;
-    two_sum_pair(hi, lo, p2, __fmaf_rn(x, x, -p2));
-  } else if (ax != 0.0f) {
-    const double d = static_cast<double>(x);
-    dx = __dadd_rn(dx, __dmul_rn(d, d));
-  }
+// One tail element, given as an fp32 bit pattern `f` (a bf16 element in the
+// high half): counted in nf if non-finite; its square added exactly to the
+// float pair (hi, lo) -- the fp32 product and its FMA residual, by TwoSum --
+// when |x| is 0 or lies in [2^-40, 2^56] (the residual is not subnormal, and
+// a lane's 8 squares add at most 2^115); any other finite value sets `odd`,
+// and the caller adds it in fp64 (rare).  No branch: the common case stays
+// off GB300's narrow fp64 pipe and the warp does not diverge.
+__device__ __forceinline__ void tail_elem(uint32_t f, uint32_t& nf, float& hi, float& lo, bool& odd) {
+  const bool nonfinite = (f & 0x7F800000u) == 0x7F800000u;
+  const float ax = fabsf(__uint_as_float(f));
+  const bool fast = ax == 0.0f || (ax >= 0x1p-40f && ax <= 0x1p56f);  // false for NaN and Inf
+  nf += nonfinite ? 1u : 0u;
+  odd |= !fast && !nonfinite;
+  const float x = fast ? __uint_as_float(f) : 0.0f;
+  const float p2 = x * x;
+  two_sum_pair(hi, lo, p2, __fmaf_rn(x, x, -p2));
 }
 
-// Adds one segment slot (see seg_value) to the float pair (hi, lo), or to dx
-// in fp64 if it is in the tagged fp64 form or its sum is 2^90 or more (rare):
-// a lane's float pair then stays below 2^119 for any chunk of fewer than 2^47
-// bytes, tail squares included, and the 32-lane tree cannot overflow.
-__device__ __forceinline__ void add_slot(uint64_t bits, float& hi, float& lo, double& dx) {
-  const float bh = __uint_as_float(static_cast<uint32_t>(bits >> 32));
-  const float bl = __uint_as_float(static_cast<uint32_t>(bits));
-  if (bits >> 63)
-    dx += -__longlong_as_double(static_cast<long long>(bits));
-  else if (bh < 0x1p90f)
-    two_sum_pair(hi, lo, bh, bl);
-  else
-    dx += static_cast<double>(bh) + static_cast<double>(bl);
+// The fp64 share of a tail element that tail_elem left out (0 for the rest).
+__device__ __forceinline__ double tail_elem_odd(uint32_t f) {
+  const float ax = fabsf(__uint_as_float(f));
+  const bool fast = ax == 0.0f || (ax >= 0x1p-40f && ax <= 0x1p56f);
+  if (fast || (f & 0x7F800000u) == 0x7F800000u) return 0.0;
+  const double d = static_cast<double>(__uint_as_float(f));
+  return __dmul_rn(d, d);
+}
+
+// Adds a pair-form segment slot (see seg_value) whose sum is below 2^90 to
+// the float pair (hi, lo); any other slot (tagged fp64 form, or 2^90 or more,
+// both rare) sets `odd`, and the caller adds it in fp64.  A lane's float pair
+// then stays below 2^119 for any chunk of fewer than 2^47 bytes, tail squares
+// included, and the 32-lane tree cannot overflow.
+__device__ __forceinline__ bool slot_fast(uint64_t bits) {
+  return !(bits >> 63) && __uint_as_float(static_cast<uint32_t>(bits >> 32)) < 0x1p90f;
+}
+__device__ __forceinline__ void add_slot(uint64_t bits, float& hi, float& lo, bool& odd) {
+  const bool fast = slot_fast(bits);
+  odd |= !fast;
+  two_sum_pair(hi, lo, fast ? __uint_as_float(static_cast<uint32_t>(bits >> 32)) : 0.0f,
+               fast ? __uint_as_float(static_cast<uint32_t>(bits)) : 0.0f);
+}
+__device__ __forceinline__ double slot_odd(uint64_t bits) {
+  if (slot_fast(bits)) return 0.0;
+  if (bits >> 63) return -__longlong_as_double(static_cast<long long>(bits));
+  return static_cast<double>(__uint_as_float(static_cast<uint32_t>(bits >> 32))) +
+         static_cast<double>(__uint_as_float(static_cast<uint32_t>(bits)));
 }
 
 __device__ __forceinline__ void prefetch_l1(const void* q) { asm volatile("prefetch.global.L1 [%0];" ::"l"(q)); }
@@ -254,15 +260,22 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
                        (tdst == nullptr || ((reinterpret_cast<uintptr_t>(tdst) + tail) & 3u) == 0);
     uint32_t w[4] = {0u, 0u, 0u, 0u};
     if (tail != 0) {
+      if (wordy) {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int32_t t = 4 * (32 * q + static_cast<int32_t>(lane)) - z;  // the word's offset in the tail
-        if (wordy && t >= 0) {
-          w[q] = __ldg(reinterpret_cast<const uint32_t*>(tsrc + t));
-        } else if (t > -4) {
+        for (int q = 0; q < 4; ++q) {
+          const int32_t t = 4 * (32 * q + static_cast<int32_t>(lane)) - z;  // the word's offset in the tail
+          if (t >= 0) w[q] = __ldg(reinterpret_cast<const uint32_t*>(tsrc + t));
+        }
+      }
+      if (!wordy || (tail & 3u) != 0) {  // byte by byte: every word, or the partial first one
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            if (t + j >= 0) w[q] |= static_cast<uint32_t>(__ldg(tsrc + (t + j))) << (8 * j);
+        for (int q = 0; q < 4; ++q) {
+          const int32_t t = 4 * (32 * q + static_cast<int32_t>(lane)) - z;
+          if (t > -4 && (!wordy || t < 0)) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              if (t + j >= 0) w[q] |= static_cast<uint32_t>(__ldg(tsrc + (t + j))) << (8 * j);
+          }
         }
       }
     }
@@ -297,15 +310,22 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
     }
     // pack and unpack copy the tail (before the body's CRC is folded into it)
     if (tdst != nullptr && tail != 0) {
+      if (wordy) {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int32_t t = 4 * (32 * q + static_cast<int32_t>(lane)) - z;
-        if (wordy && t >= 0) {
-          *reinterpret_cast<uint32_t*>(tdst + t) = w[q];
-        } else if (t > -4) {
+        for (int q = 0; q < 4; ++q) {
+          const int32_t t = 4 * (32 * q + static_cast<int32_t>(lane)) - z;
+          if (t >= 0) *reinterpret_cast<uint32_t*>(tdst + t) = w[q];
+        }
+      }
+      if (!wordy || (tail & 3u) != 0) {
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            if (t + j >= 0) tdst[t + j] = static_cast<uint8_t>(w[q] >> (8 * j));
+        for (int q = 0; q < 4; ++q) {
+          const int32_t t = 4 * (32 * q + static_cast<int32_t>(lane)) - z;
+          if (t > -4 && (!wordy || t < 0)) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              if (t + j >= 0) tdst[t + j] = static_cast<uint8_t>(w[q] >> (8 * j));
+          }
         }
       }
     }
@@ -318,9 +338,12 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
     uint32_t nf_lane = 0;  // this lane's share of the non-finite count
     uint64_t carry = 0;
     if (rec_mul) {
-      if (lane < n_recs) {
-        raw = mul0 == kOne ? rec0.crc : gmul(rec0.crc, mul0);
-        nf_lane = rec0.nonfinite;
+      raw = rec0.crc;  // zero past the chunk's records
+      nf_lane = rec0.nonfinite;
+      const bool shift = lane < n_recs && mul0 != kOne;
+      if (__any_sync(kFull, shift)) {
+        const uint32_t r = gmul(rec0.crc, mul0);
+        if (shift) raw = r;
       }
       for (int64_t i = lane + 32; i < n_recs; i += 32) {
         const Record rec = p.recs[first_rec + i];
@@ -361,20 +384,39 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
     double sq = 0.0;
     if (values) {
       float hi = 0.0f, lo = 0.0f;
-      double dx = 0.0;
-      if (lane < n_seg) add_slot(slot0, hi, lo, dx);
-      for (uint64_t k = lane + 32; k < n_seg; k += 32)
-        add_slot(reinterpret_cast<const uint64_t*>(p.segs + cd.seg_base)[k], hi, lo, dx);
+      bool odd = false;
+      const uint64_t* seg_slots = reinterpret_cast<const uint64_t*>(p.segs + cd.seg_base);
+      add_slot(slot0, hi, lo, odd);  // zero past the body's segments
+      for (uint64_t k = lane + 32; k < n_seg; k += 32) add_slot(seg_slots[k], hi, lo, odd);
+      const bool f32 = cd.dtype == kDtF32;
       if (tail != 0) {
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          if (cd.dtype == kDtF32) {
-            tail_elem(kDtF32, w[q], nf_lane, hi, lo, dx);
+          if (f32) {
+            tail_elem(w[q], nf_lane, hi, lo, odd);
           } else {
-            tail_elem(kDtBf16, w[q] & 0xFFFFu, nf_lane, hi, lo, dx);
-            tail_elem(kDtBf16, w[q] >> 16, nf_lane, hi, lo, dx);
+            tail_elem(w[q] << 16, nf_lane, hi, lo, odd);
+            tail_elem(w[q] & 0xFFFF0000u, nf_lane, hi, lo, odd);
           }
         }
+      }
+      double dx = 0.0;  // the values left out of the float pairs, in fp64 (rare)
+      if (__any_sync(kFull, odd)) {
+        if (odd) {
+          dx = slot_odd(slot0);
+          for (uint64_t k = lane + 32; k < n_seg; k += 32) dx += slot_odd(seg_slots[k]);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            if (f32) {
+              dx += tail_elem_odd(w[q]);
+            } else {
+              dx += tail_elem_odd(w[q] << 16);
+              dx += tail_elem_odd(w[q] & 0xFFFF0000u);
+            }
+          }
+        }
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) dx += __shfl_down_sync(kFull, dx, m);
       }
       // lanes at or past `active` hold zeros: tree levels that would only add
       // them are skipped (adding (0, 0) changes no bit of the pair)
@@ -385,10 +427,6 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
           const float oh = __shfl_down_sync(kFull, hi, m), ol = __shfl_down_sync(kFull, lo, m);
           two_sum_pair(hi, lo, oh, ol);
         }
-      }
-      if (__any_sync(kFull, dx != 0.0)) {
-#pragma unroll
-        for (int m = 16; m >= 1; m >>= 1) dx += __shfl_down_sync(kFull, dx, m);
       }
       sq = (static_cast<double>(hi) + static_cast<double>(lo)) + dx;
     }
@@ -406,11 +444,11 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
       const bool fold = (tail & 3u) == 0;
       if (fold) {
         const uint32_t i0 = static_cast<uint32_t>(z) >> 2;  // the window word holding the tail's first byte
-        if (lane == (i0 & 31u)) {
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            if (static_cast<uint32_t>(q) == (i0 >> 5)) w[q] ^= raw;
-        }
+        const uint32_t fx = lane == (i0 & 31u) ? raw : 0u;
+        w[0] ^= (i0 >> 5) == 0 ? fx : 0u;
+        w[1] ^= (i0 >> 5) == 1 ? fx : 0u;
+        w[2] ^= (i0 >> 5) == 2 ? fx : 0u;
+        w[3] ^= (i0 >> 5) == 3 ? fx : 0u;
       }
       const uint32_t H = mul_x32k(6, mul_x32k(5, w[0]) ^ w[1]) ^ (mul_x32k(5, w[2]) ^ w[3]);
       const uint32_t joined = __reduce_xor_sync(kFull, lane_mul(LM, H));
