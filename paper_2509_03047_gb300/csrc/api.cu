@@ -286,6 +286,7 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
       uint32_t cls;
       uint64_t list_off;
       std::vector<uint64_t> seg_start;
+      std::vector<uint64_t> cost;  // cost[s]: estimated cost of segments [0, s)
     };
     std::vector<Cls> cl;
     for (uint32_t cls = 0; cls < 6; ++cls) {
@@ -296,9 +297,15 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
       for (uint64_t c = bi.c_begin; c < bi.c_end; ++c)
         if (chunks[c].sweep_class == cls && chunks[c].len >= static_cast<uint64_t>(kBlockBytes))
           lists.push_back(static_cast<uint32_t>(c));
+      q.cost.push_back(0);
       for (size_t i = q.list_off; i < lists.size(); ++i) {
         const ChunkDesc& d = chunks[lists[i]];
-        for (uint64_t j = 0; j < d.len / kBlockBytes; j += kSegBlocks) q.seg_start.push_back(d.blk_begin + j);
+        const uint64_t nb = d.len / kBlockBytes;
+        for (uint64_t j = 0; j < nb; j += kSegBlocks) {
+          q.seg_start.push_back(d.blk_begin + j);
+          const uint64_t blocks = std::min<uint64_t>(kSegBlocks, nb - j);
+          q.cost.push_back(q.cost.back() + seg_cost(blocks, j == 0));
+        }
       }
       q.seg_start.push_back(class_blocks[cls]);
       cl.push_back(std::move(q));
@@ -364,8 +371,12 @@ cudaError_t build_decomp(const std::vector<ChunkDesc>& base, const std::vector<u
         }
         return wd;
       };
+      // the warps' ranges: the first n_fix segments cut by estimated cost
+      std::vector<uint64_t> bnd(Wq + 1);
+      const std::vector<uint64_t>& cost = cl[q].cost;
+      split_ranges([&](uint64_t i) { return cost[i]; }, n_fix, Wq, bnd.data());
       for (uint64_t w = 0; w < Wq; ++w) {
-        const WarpDesc wd = range(seg_start[n_fix * w / Wq], seg_start[n_fix * (w + 1) / Wq]);
+        const WarpDesc wd = range(seg_start[bnd[w]], seg_start[bnd[w + 1]]);
         if (mixed)
           warps[warp_base + slot[q * W + w]] = wd;
         else

@@ -65,6 +65,8 @@ struct HostTables {
   WarpDesc warps[kMaxWarps];
   uint64_t rec_nblk[kMaxRecs];
   uint64_t seg_start[kMaxSegs + 1];  // per class: block where each segment starts
+  uint64_t seg_cost[kMaxSegs + 1];   // per class: estimated cost of its segments before each
+  uint64_t bnd[kMaxWarps + 1];       // per class: the segment where each warp's range starts
   uint32_t slot[kClasses * kMaxWarps];  // per class: launch-warp index of its j-th warp
 };
 HostTables g_host;
@@ -198,15 +200,21 @@ extern "C" fr_status fr_fingerprint_static(const fr_tensor* tensors, uint64_t n_
     const uint32_t* list = h.lists + list_off;
     // warp ranges start on 16 KiB segment boundaries (see layout.h)
     uint64_t n_class_segs = 0;
+    h.seg_cost[0] = 0;
     for (uint64_t i = list_off; i < n_lists; ++i) {
       const ChunkDesc& d = h.chunks[h.lists[i]];
       const uint64_t nb = d.len / kBlockBytes;
-      for (uint64_t j = 0; j < nb; j += kSegBlocks) h.seg_start[n_class_segs++] = d.blk_begin + j;
+      for (uint64_t j = 0; j < nb; j += kSegBlocks) {
+        h.seg_start[n_class_segs] = d.blk_begin + j;
+        h.seg_cost[n_class_segs + 1] = h.seg_cost[n_class_segs] + seg_cost(std::min<uint64_t>(kSegBlocks, nb - j), j == 0);
+        ++n_class_segs;
+      }
     }
     h.seg_start[n_class_segs] = blk;
+    split_ranges([&](uint64_t s) { return h.seg_cost[s]; }, n_class_segs, Wq, h.bnd);
     uint64_t k = 0;
     for (uint64_t w = 0; w < Wq; ++w) {
-      const uint64_t b0 = h.seg_start[n_class_segs * w / Wq], b1 = h.seg_start[n_class_segs * (w + 1) / Wq];
+      const uint64_t b0 = h.seg_start[h.bnd[w]], b1 = h.seg_start[h.bnd[w + 1]];
       WarpDesc& wd = h.warps[h.slot[q * kMaxWarps + w]];
       std::memset(&wd, 0, sizeof wd);
       wd.blk_begin = b0;

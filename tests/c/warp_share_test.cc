@@ -1,5 +1,6 @@
 // warp_share_test.cc -- checks the rule that shares one sweep launch's warps
-// among the element-type/alignment classes (csrc/warp_share.h), on the host.
+// among the element-type/alignment classes, and the cost-weighted cut of a
+// class into warp ranges (csrc/warp_share.h), on the host.
 // Exits 0 and prints "warp_share ok" when every check holds.
 #include <cmath>
 #include <cstdio>
@@ -57,7 +58,50 @@ static int check(const std::vector<double>& cost, int n_ctas, int wpc) {
   return 0;
 }
 
+// split_ranges: boundaries are monotone, span [0, n], and each is the last
+// one whose cost prefix is at most its share of the total; unit costs give
+// floor(n * w / Wq).
+static int check_split(const std::vector<uint64_t>& seg, uint64_t Wq) {
+  const uint64_t n = seg.size();
+  std::vector<uint64_t> pre(n + 1, 0);
+  for (uint64_t s = 0; s < n; ++s) pre[s + 1] = pre[s] + seg[s];
+  std::vector<uint64_t> bnd(Wq + 1);
+  split_ranges([&](uint64_t s) { return pre[s]; }, n, Wq, bnd.data());
+  EXPECT(bnd[0] == 0 && bnd[Wq] == n);
+  for (uint64_t w = 0; w <= Wq; ++w) {
+    if (w > 0) EXPECT(bnd[w] >= bnd[w - 1]);
+    const unsigned __int128 target = static_cast<unsigned __int128>(pre[n]) * w;
+    EXPECT(static_cast<unsigned __int128>(pre[bnd[w]]) * Wq <= target || w == 0);
+    EXPECT(bnd[w] == n || static_cast<unsigned __int128>(pre[bnd[w] + 1]) * Wq > target || w == 0);
+  }
+  return 0;
+}
+
 int main() {
+  // split_ranges on unit costs is the equal-count split
+  for (uint64_t n : {0ull, 1ull, 7ull, 1000ull, 4099ull})
+    for (uint64_t Wq : {1ull, 3ull, 16ull, 2432ull}) {
+      std::vector<uint64_t> pre(n + 1);
+      for (uint64_t s = 0; s <= n; ++s) pre[s] = s;
+      std::vector<uint64_t> bnd(Wq + 1);
+      split_ranges([&](uint64_t s) { return pre[s]; }, n, Wq, bnd.data());
+      for (uint64_t w = 0; w <= Wq; ++w) EXPECT(bnd[w] == n * w / Wq);
+    }
+  // uneven costs: chunk starts, partial segments, zero-cost runs
+  {
+    std::vector<uint64_t> seg;
+    uint32_t x = 12345;
+    for (int i = 0; i < 5000; ++i) {
+      x = x * 1103515245u + 12345u;
+      const uint64_t blocks = 1 + (x >> 16) % 32;
+      seg.push_back(seg_cost(blocks, (x >> 8) % 5 == 0));
+    }
+    for (uint64_t Wq : {1ull, 2ull, 152ull, 2432ull, 6000ull})
+      if (check_split(seg, Wq)) return 1;
+    if (check_split({0, 0, 5, 0, 0, 7, 0}, 4)) return 1;
+  }
+  EXPECT(seg_cost(32, true) > seg_cost(32, false) && seg_cost(32, false) > seg_cost(1, false));
+
   // a Llama shard: bf16 weights (1/7 of the bytes, weighted 1.25) and fp32 state
   const double bf16 = 1.0 * block_weight(kDtBf16, kShareFingerprint);
   const double f32 = 6.0 * block_weight(kDtF32, kShareFingerprint);

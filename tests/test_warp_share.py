@@ -2,7 +2,9 @@
 alignment classes (csrc/warp_share.h), compiled with the host C++ compiler
 and checked by tests/c/warp_share_test.cc: warp counts sum to the launch,
 follow the weighted block counts, give every class at least one warp, and
-every CTA gets an even share of every class.  No GPU."""
+every CTA gets an even share of every class; within a class the ranges are
+cut by estimated segment cost (monotone boundaries covering every segment,
+the equal-count split for unit costs).  No GPU."""
 import os
 import shutil
 import subprocess
