@@ -21,8 +21,9 @@
 //    recovered to second order by a TwoSum whose low term is a second FMA
 //    (two_sum_sq), then flushed into fp64.  A 16 KiB segment whose running
 //    sum is not finite (NaN/Inf input, or overflow) or is tiny with non-zero
-//    input is redone element by element in fp64 from a reload of its 16-byte
-//    units, so the fast path never needs a per-element test.
+//    input is redone element by element, exactly, from a reload of its
+//    16-byte units (slow_span), so the fast path never needs a per-element
+//    test.
 //
 // No tensor cores: nothing here is a contraction.  One CTA per SM, with a warp
 // count per mode (the 128 KiB of lane-replicated tables fill most of shared
@@ -313,36 +314,52 @@ struct Exact {
   uint32_t nonfinite;
 };
 
-// Exact per-element fallback for this lane's units of blocks [b0, b1).
+// Exact per-element fallback for this lane's units of blocks [b0, b1):
+// non-finite elements are counted; each finite square is added exactly --
+// for |x| in [2^-40, 2^56] as its fp32 product and FMA residual into an
+// unevaluated float pair by TwoSum, else (tiny or huge values, rare) in fp64,
+// where the square of an fp32 value is exact.  Its error, under n^2 u^2 of
+// the sum for the n elements of a lane, is far inside the sums' bound.  The
+// segment was just swept (its lines are mostly in L2); the lane first
+// prefetches all its units into L1, so the reloads do not wait for L2 one by
+// one, and the float pair keeps the arithmetic off GB300's narrow fp64 pipe.
+// (Loading the units in register batches instead makes the compiler spill in
+// the hot loop that calls this.)
 template <int DT, int AL>
 __device__ __noinline__ Exact slow_span(const uint8_t* sp, uint64_t b0, uint64_t b1) {
+  for (uint64_t b = b0; b < b1; ++b) asm volatile("prefetch.global.L1 [%0];" ::"l"(sp + b * kBlockBytes));
+  float hi = 0.0f, lo = 0.0f;
   double d = 0.0;
   uint32_t nonfinite = 0;
   for (uint64_t b = b0; b < b1; ++b) {
     const uint4 v = ld_unit<AL>(sp + b * kBlockBytes);
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
     for (int j = 0; j < 4; ++j) {
-      if (DT == kDtF32) {
-        if ((w[j] & 0x7F800000u) == 0x7F800000u) {
+#pragma unroll
+      for (int h = 0; h < (DT == kDtF32 ? 1 : 2); ++h) {
+        const uint32_t f = DT == kDtF32 ? w[j] : (h == 0 ? w[j] << 16 : w[j] & 0xFFFF0000u);
+        if ((f & 0x7F800000u) == 0x7F800000u) {
           ++nonfinite;
-        } else {
-          const double x = static_cast<double>(__uint_as_float(w[j]));
-          d = __dadd_rn(d, __dmul_rn(x, x));
+          continue;
         }
-      } else {
-        for (int h = 0; h < 2; ++h) {
-          const uint32_t bits = (w[j] >> (16 * h)) & 0xFFFFu;
-          if ((bits & 0x7F80u) == 0x7F80u) {
-            ++nonfinite;
-          } else {
-            const double x = static_cast<double>(__uint_as_float(bits << 16));
-            d = __dadd_rn(d, __dmul_rn(x, x));
-          }
+        const float x = __uint_as_float(f);
+        const float ax = fabsf(x);
+        if (ax >= 0x1p-40f && ax <= 0x1p56f) {
+          const float p2 = x * x;
+          const float e = __fmaf_rn(x, x, -p2);
+          const float t = hi + p2;
+          const float z = t - hi;
+          lo += ((hi - (t - z)) + (p2 - z)) + e;
+          hi = t;
+        } else if (ax != 0.0f) {
+          const double xd = static_cast<double>(x);
+          d = __dadd_rn(d, __dmul_rn(xd, xd));
         }
       }
     }
   }
-  return Exact{d, nonfinite};
+  return Exact{(static_cast<double>(hi) + static_cast<double>(lo)) + d, nonfinite};
 }
 
 // Whether this lane's units of blocks [b0, b1) hold only (signed) zeros.
