@@ -9,11 +9,14 @@
 //      non-finite counts, and adds the body's 16 KiB segment sums of squares
 //      in an order fixed by segment index (so the result does not depend on
 //      the plan);
-//   2. handles the chunk's tail (len % 512 bytes, if any): lane l takes the
-//      16 bytes ending 16 * (31 - l) bytes before its end, copies them for
-//      pack/unpack, sums their squares, and CRCs them a word at a time with
-//      the body's raw CRC folded into the tail's first word (which continues
-//      the body's CRC through the tail without shifting it);
+//   2. handles the chunk's tail (len % 512 bytes, if any) as the end of a
+//      512-byte window with leading zeros, window word i in lane i % 32:
+//      copies it for pack/unpack (whole words when aligned), adds its squares
+//      to the lanes' segment sums before one lane tree, and CRCs it with the
+//      body's raw CRC folded into the tail's first word (which continues the
+//      body's CRC through the tail without shifting it): each lane combines
+//      its words by constant multiplies, takes its lane's shift from a
+//      shared-memory table, and the lanes are XORed;
 //   3. applies CRC-32C's preset and final XOR:
 //      crc = raw ^ 0xFFFFFFFF * x^(8 len) ^ 0xFFFFFFFF;
 //   4. fingerprint: writes the table entry; pack: writes the 64-byte header,
