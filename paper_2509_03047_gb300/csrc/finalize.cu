@@ -49,21 +49,13 @@ constexpr int kFinThreads = kFinWarps * 32;
 constexpr unsigned kFull = 0xFFFFFFFFu;
 
 __device__ const PowTables g_pow = make_pow_tables();
-// Byte tables for multiplying by the constants x^(32 * 2^k), k = 0..6
-// (x^32 ... x^2048); the tail's CRC uses x^1024 and x^2048.
-struct ConstMulTables {
-  ByteTables4 m[7];
-};
-__host__ __device__ constexpr ConstMulTables make_const_mul_tables() {
-  ConstMulTables t{};
-  for (int k = 0; k < 7; ++k) t.m[k] = make_mul_tables(gf_xpow(32ull << k));
-  return t;
-}
-__device__ const ConstMulTables g_cmul = make_const_mul_tables();
+// Byte tables for multiplying by x^1024 and x^2048: a tail lane combines its
+// four window words, 32 words apart, with them.
+__device__ const ByteTables4 g_x1024 = make_mul_tables(gf_xpow(1024));
+__device__ const ByteTables4 g_x2048 = make_mul_tables(gf_xpow(2048));
 
-// a * x^(32 * 2^k) mod P.
-__device__ __forceinline__ uint32_t mul_x32k(int k, uint32_t a) {
-  const ByteTables4& T = g_cmul.m[k];
+// a * m mod P, T being the byte tables of the constant m.
+__device__ __forceinline__ uint32_t mul_const(const ByteTables4& T, uint32_t a) {
   return (__ldg(&T.t[0][a & 255u]) ^ __ldg(&T.t[1][(a >> 8) & 255u])) ^
          (__ldg(&T.t[2][(a >> 16) & 255u]) ^ __ldg(&T.t[3][a >> 24]));
 }
@@ -453,7 +445,7 @@ __global__ void __launch_bounds__(kFinThreads, FR_FIN_MINB) finalize_kernel(Fina
         w[2] ^= (i0 >> 5) == 2 ? fx : 0u;
         w[3] ^= (i0 >> 5) == 3 ? fx : 0u;
       }
-      const uint32_t H = mul_x32k(6, mul_x32k(5, w[0]) ^ w[1]) ^ (mul_x32k(5, w[2]) ^ w[3]);
+      const uint32_t H = mul_const(g_x2048, mul_const(g_x1024, w[0]) ^ w[1]) ^ (mul_const(g_x1024, w[2]) ^ w[3]);
       const uint32_t joined = __reduce_xor_sync(kFull, lane_mul(LM, H));
       raw = (fold || raw == 0) ? joined : (shift_bytes(raw, tail) ^ joined);
     }

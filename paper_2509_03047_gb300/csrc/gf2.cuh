@@ -97,25 +97,6 @@ __host__ __device__ constexpr ByteTables4 make_mul_tables(uint32_t m) {
   return out;
 }
 
-struct ByteTable {
-  uint32_t t[256];
-};
-
-// t[b] = b * x^8: the classic one-byte-at-a-time table.
-__host__ __device__ constexpr ByteTable make_byte_table() {
-  ByteTable out{};
-  const uint32_t x8 = gf_xpow(8);
-  uint32_t bit[8] = {};
-  for (int j = 0; j < 8; ++j) bit[j] = gf_mulmod(1u << j, x8);
-  for (int b = 0; b < 256; ++b) {
-    uint32_t v = 0;
-    for (int j = 0; j < 8; ++j)
-      if (b & (1 << j)) v ^= bit[j];
-    out.t[b] = v;
-  }
-  return out;
-}
-
 // Powers for shifting a raw CRC by n bytes: x^(8n) = prod_k p[k][byte k of n].
 constexpr int kPowBytes = 6;  // n < 2^48
 struct PowTables {
