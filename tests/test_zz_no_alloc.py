@@ -13,7 +13,8 @@ import torch
 
 from paper_2509_03047_gb300 import synth
 
-from gpu_helpers import Guarded, assert_tables_match, odd_tensors, table_np
+import oracle
+from gpu_helpers import Guarded, assert_tables_match, host_bytes, odd_tensors, table_np
 
 pytestmark = pytest.mark.gpu
 
@@ -45,6 +46,9 @@ def test_static_entry_point_matches_plan_on_three_calls_in_a_row():
         got = _static_table(tensors, chunk)
         assert got.numel() == want.numel()
         assert_tables_match(table_np(got), table_np(want), "static vs plan")
+        # and directly against the oracle, every entry
+        dtypes = [fr.fr_dtype_of(t) for t in tensors]
+        assert_tables_match(table_np(got), oracle.fingerprint(host_bytes(tensors), dtypes, chunk), "static vs oracle")
 
 
 def test_static_entry_point_rejects_inputs_beyond_its_limit():
