@@ -4,8 +4,9 @@
 // The planner turns a tensor list into the device tables of layout.h:
 // per-tensor chunks, the packed layout, and one or two "decompositions" of the
 // chunk bodies into per-warp work.  The whole-state decomposition cuts each
-// (element type, alignment) class's block stream into equal ranges for the
-// warps of every SM; a batched plan also cuts the chunks into consecutive
+// (element type, alignment) class's block stream into ranges of equal
+// estimated cost for the warps of every SM; a batched plan also cuts the
+// chunks into consecutive
 // batches of about equal bytes, each decomposed over half the SMs, so that a
 // replica's pack of batch b+1 and a restarted rank's unpack of batch b can run
 // side by side (a sweep CTA holds most of an SM's shared memory, so two
@@ -238,8 +239,8 @@ void free_device(fr_plan p) {
 
 // Cut the chunks [bounds[b], bounds[b+1]) of every batch b into sweep work for
 // `n_ctas` CTAs: per batch and class, the class's 16 KiB segments in chunk
-// order are split into equal runs, one per warp, and every (warp, chunk)
-// overlap gets one record.  Records are numbered batch by batch, class
+// order are split into runs of equal estimated cost (split_ranges), one per
+// warp, and every (warp, chunk) overlap gets one record.  Records are numbered batch by batch, class
 // by class, so each chunk's records are consecutive.  `min_recs`: record slots
 // to allocate at least (list-mode calls use one slot per listed chunk).
 // Plain: every class gets all n_ctas * warps_per_cta warps (one launch per

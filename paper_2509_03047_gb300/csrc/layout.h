@@ -5,9 +5,10 @@
 // "tail" of len % 512 bytes.  Chunks fall into sweep classes by element type
 // and by whether their tensor is 16-byte aligned.  The bodies of a class's
 // chunks, concatenated in chunk order, form one block stream that is cut into
-// equal ranges, one per warp the call's sweep launch gives that class
-// (warp_share.h), so a class's warps move equal bytes whatever the tensor
-// sizes.  A warp's range overlaps
+// ranges of equal estimated cost (bytes, segment ends, chunk starts), one per
+// warp the call's sweep launch gives that class (warp_share.h), so a class's
+// warps take about equal time whatever the tensor sizes.  A warp's range
+// overlaps
 // one or more chunks; each overlap is a "piece" and produces one record (raw
 // CRC, non-finite count).  Warp ranges start on segment boundaries.
 // The records of a chunk are consecutive and in order.  The finalize kernel
