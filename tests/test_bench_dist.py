@@ -68,3 +68,5 @@ def test_reference_arm_prints_on_rank_zero_only():
     line = json.loads(outs[1])
     assert line["impl"] == "reference" and line["unit"] == "GB/s" and line["value"] > 0
     assert line["cpu_baseline"]["kind"] == "oracle" and line["e2e"]["h2d_bytes_per_step"] == 0
+    # the oracle arm maps the oracle only, never the product library
+    assert line["native_libraries"] == ["oracle/liboracle.so"]
